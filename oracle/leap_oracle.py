@@ -1,0 +1,334 @@
+"""Plain, slow fp64 CPU oracle for the LEAP GRPO-loss hot path.
+
+TEST INFRASTRUCTURE ONLY.  Nothing on the product path may import this module:
+only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` use it.  It shares no code with the
+CUDA library (``paper_2608_01804_gb300``) and imports nothing from it.
+
+Every function follows the paper (LEAP: Lean Environment-Feedback via Adaptive
+Pruning, arXiv 2608.01804) in its own order and notation, in float64, with
+numpy used only for whole-array primitives (max, exp, log, sum, matmul).
+Where the paper is silent the function states the reading it takes; the same
+readings are listed in the design doc.
+
+Pins (what checks this oracle against something other than itself) live in
+``tests/test_oracle_*.py``.  No function here is "parity unpinned".
+
+Conventions shared with the library's contract (not the paper's):
+  * outcomes are per rollout: ``pass_turn`` = 1-based turn of the first passing
+    verification (0 = never passed), ``num_turns`` = generated turns T_i;
+  * a rollout whose outcome fields are out of range is treated as a failure
+    (r = 0) that contributes no tokens (T_eff = 0), and is reported in the
+    returned ``bad_outcome`` mask;
+  * a token whose id lies outside [0, V) is treated as masked (w = 0) and is
+    reported in ``bad_id``;
+  * rows with w == 0 are not read: their logp, lse, ell and dlogits are 0.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+
+AGG_SEQ_MEAN_TOKEN_MEAN = 0
+AGG_TOKEN_MEAN = 1
+ADVNORM_GRPO_STD = 0
+ADVNORM_NONE = 1
+
+
+# ---------------------------------------------------------------------------
+# Sec. 3.1 (DCP), Eq. 1-2, and Sec. 3.2 (rank tiers), Eq. 4 and the tier rule.
+# ---------------------------------------------------------------------------
+def tiers_and_gate(pass_turn, num_turns, M, tau_min, tau_max, gate_in=None):
+    """Failure count, DCP gate, rank tier r and effective turn count per rollout.
+
+    Eq. 1: N_fail(q) = sum_i I(o_i failed).  Reading: "failed" is judged on the
+    first turn, because the gate decides whether turn 2 is generated at all.
+    Eq. 2: G(q) = 1 iff tau_min <= N_fail <= tau_max (both bounds inclusive).
+    Tier rule (Sec. 3.2): pass at turn m -> r = M - m + 1; never passed -> r = 0.
+    A gated-off group (G(q) = 0) never ran turns after the first, so its
+    outcomes are truncated to turn 1: r = M on a first-turn pass, else 0, and
+    T_eff = 1.  ``gate_in`` (if given) replaces Eq. 2 with a recorded gate.
+
+    Arrays are [num_groups, G].  Returns (n_fail, gate, r, T_eff, bad_outcome).
+    """
+    pass_turn = np.asarray(pass_turn, dtype=np.int64)
+    num_turns = np.asarray(num_turns, dtype=np.int64)
+    num_groups, G = pass_turn.shape
+
+    bad = np.zeros((num_groups, G), dtype=bool)
+    n_fail = np.zeros(num_groups, dtype=np.int64)
+    gate = np.zeros(num_groups, dtype=np.uint8)
+    r = np.zeros((num_groups, G), dtype=np.int64)
+    T_eff = np.zeros((num_groups, G), dtype=np.int64)
+
+    for g in range(num_groups):
+        for i in range(G):
+            m, T = pass_turn[g, i], num_turns[g, i]
+            if m < 0 or m > M or T < 1 or T > M or (m >= 1 and m > T):
+                bad[g, i] = True
+        # Eq. 1 over first-turn outcomes (a malformed rollout counts as failed).
+        for i in range(G):
+            if bad[g, i] or pass_turn[g, i] != 1:
+                n_fail[g] += 1
+        if gate_in is not None:
+            gate[g] = 1 if gate_in[g] != 0 else 0
+        else:
+            gate[g] = 1 if (tau_min <= n_fail[g] <= tau_max) else 0   # Eq. 2
+        for i in range(G):
+            if bad[g, i]:
+                r[g, i], T_eff[g, i] = 0, 0
+                continue
+            m = pass_turn[g, i]
+            if gate[g] == 0:
+                r[g, i] = M if m == 1 else 0
+                T_eff[g, i] = 1
+            else:
+                r[g, i] = (M - m + 1) if m >= 1 else 0
+                T_eff[g, i] = num_turns[g, i]
+    return n_fail, gate, r, T_eff, bad
+
+
+# ---------------------------------------------------------------------------
+# Sec. 3.2, Eq. 5: the complete pairwise tournament, literally.
+# ---------------------------------------------------------------------------
+def tournament(r):
+    """N_worse(o_i) = #{j != i : r_i > r_j},  N_better(o_i) = #{j != i : r_i < r_j}.
+
+    Strict inequalities: a tie counts in neither.  This is the O(G^2) double
+    loop of Eq. 5 (vectorised over j for speed; the comparison is the same).
+    """
+    r = np.asarray(r, dtype=np.int64)
+    num_groups, G = r.shape
+    n_worse = np.zeros((num_groups, G), dtype=np.int64)
+    n_better = np.zeros((num_groups, G), dtype=np.int64)
+    for i in range(G):
+        ri = r[:, i:i + 1]
+        others = np.ones(G, dtype=bool)
+        others[i] = False
+        n_worse[:, i] = np.sum((ri > r) & others, axis=1)
+        n_better[:, i] = np.sum((ri < r) & others, axis=1)
+    return n_worse, n_better
+
+
+def tournament_reward(n_worse, n_better, G):
+    """Eq. 6: R_i = (N_worse(o_i) - N_better(o_i)) / (G - 1), in [-1, 1]."""
+    if G < 2:
+        raise ValueError("Eq. 6 divides by G - 1: G must be at least 2")
+    return (np.asarray(n_worse, np.float64) - np.asarray(n_better, np.float64)) / (G - 1)
+
+
+def grpo_advantage(R, eps_std=1e-6, norm=ADVNORM_GRPO_STD, std_unbiased=True):
+    """Sec. 3.2, last step: the final advantage A_i by "the standard GRPO formulation".
+
+    Reading: A_i = (R_i - mean_g R) / (std_g R + eps_std) over the rollout group,
+    std with the (G - 1) divisor by default.  ``ADVNORM_NONE`` returns R as is.
+    """
+    R = np.asarray(R, dtype=np.float64)
+    if norm == ADVNORM_NONE:
+        return R.copy()
+    G = R.shape[1]
+    mean = R.sum(axis=1, keepdims=True) / G
+    dev = R - mean
+    ddof = 1 if std_unbiased else 0
+    std = np.sqrt((dev * dev).sum(axis=1, keepdims=True) / (G - ddof))
+    return dev / (std + eps_std)
+
+
+def turn_advantages(A, T_eff, gamma, M):
+    """Sec. 3.3: discounted per-turn advantage.
+
+    beta_i = gamma if A_i >= 0 else 1;  A_hat_{i,t} = beta_i^(T_i - t - 1) * A_i
+    for generated turns t = 0 .. T_i - 1 (T_i = the effective turn count after
+    DCP).  Turns t >= T_i get 0.  Returns [num_groups, G, M].
+    """
+    A = np.asarray(A, dtype=np.float64)
+    T_eff = np.asarray(T_eff, dtype=np.int64)
+    num_groups, G = A.shape
+    out = np.zeros((num_groups, G, M), dtype=np.float64)
+    for g in range(num_groups):
+        for i in range(G):
+            beta = gamma if A[g, i] >= 0 else 1.0
+            for t in range(T_eff[g, i]):
+                out[g, i, t] = (beta ** (T_eff[g, i] - t - 1)) * A[g, i]
+    return out
+
+
+def rank_advantages(pass_turn, num_turns, M, tau_min, tau_max, gamma,
+                    eps_std=1e-6, norm=ADVNORM_GRPO_STD, std_unbiased=True,
+                    gate_in=None):
+    """Sec. 3.1-3.3 end to end for every group: gate, tiers, tournament, R, A, A_hat."""
+    pass_turn = np.asarray(pass_turn)
+    G = pass_turn.shape[1]
+    n_fail, gate, r, T_eff, bad = tiers_and_gate(pass_turn, num_turns, M,
+                                                 tau_min, tau_max, gate_in)
+    n_worse, n_better = tournament(r)
+    R = tournament_reward(n_worse, n_better, G)
+    A = grpo_advantage(R, eps_std, norm, std_unbiased)
+    turn_adv = turn_advantages(A, T_eff, gamma, M)
+    return dict(n_fail=n_fail, gate=gate, r=r, T_eff=T_eff, bad_outcome=bad,
+                n_worse=n_worse, n_better=n_better, R=R, A=A, turn_adv=turn_adv)
+
+
+# ---------------------------------------------------------------------------
+# Sec. 3.3 (token sets M_{i,t}) and Sec. 4.1 (sample-level aggregation).
+# ---------------------------------------------------------------------------
+def rollout_token_counts(seg_offsets, seg_rollout, seg_turn, T_eff_flat):
+    """L_i = number of optimised tokens of rollout i = sum of |M_{i,t}| over t < T_eff_i.
+
+    Segments are consecutive ranges [seg_offsets[s], seg_offsets[s+1]) of the
+    packed token stream.  seg_turn < 0 (prompt, feedback, padding) or a turn at
+    or beyond T_eff (pruned by DCP) contributes nothing (Sec. 3.3: tokens
+    outside the generated turns get zero advantage and are excluded).
+    Returns (L [n], n_valid_tokens, n_valid_rollouts).
+    """
+    n = len(T_eff_flat)
+    L = np.zeros(n, dtype=np.int64)
+    for s in range(len(seg_rollout)):
+        i, t = int(seg_rollout[s]), int(seg_turn[s])
+        if t < 0 or i < 0 or i >= n:
+            continue
+        if t < T_eff_flat[i]:
+            L[i] += int(seg_offsets[s + 1]) - int(seg_offsets[s])
+    return L, int(L.sum()), int(np.count_nonzero(L))
+
+
+def token_advantages(N, seg_offsets, seg_rollout, seg_turn, turn_adv_flat, T_eff_flat,
+                     M, agg, L, n_valid_tokens, n_valid_rollouts):
+    """Per-token advantage A_hat_k and loss weight w_k.
+
+    Sec. 3.3: every token of generated turn t of rollout i carries A_hat_{i,t};
+    every other token carries 0 and weight 0.
+    Sec. 4.1 ("sample-level loss objective"), reading: each rollout's loss is
+    the mean over its own tokens, and the batch loss the mean over rollouts
+    with at least one token, so w_k = 1 / (R_valid * L_i).  TOKEN_MEAN instead
+    averages over all valid tokens: w_k = 1 / N_valid.  The normalisers are
+    global (passed in) so that shards and chunks sum to the whole.
+    """
+    adv = np.zeros(N, dtype=np.float64)
+    w = np.zeros(N, dtype=np.float64)
+    for s in range(len(seg_rollout)):
+        i, t = int(seg_rollout[s]), int(seg_turn[s])
+        if t < 0 or i < 0 or t >= T_eff_flat[i]:
+            continue
+        a, b = int(seg_offsets[s]), int(seg_offsets[s + 1])
+        adv[a:b] = turn_adv_flat[i * M + t]
+        if agg == AGG_TOKEN_MEAN:
+            w[a:b] = 1.0 / float(n_valid_tokens)
+        else:
+            w[a:b] = 1.0 / (float(n_valid_rollouts) * float(L[i]))
+    return adv, w
+
+
+# ---------------------------------------------------------------------------
+# Token log-probabilities under pi_theta (Eq. 3's surrogate needs log pi).
+# ---------------------------------------------------------------------------
+def bf16_bits_to_f64(bits):
+    """bf16 bit patterns (uint16) -> exact float64 values."""
+    u = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return u.view(np.float32).astype(np.float64)
+
+
+def f64_to_bf16_bits(x):
+    """Round float64 to the nearest bf16 (ties to even) via float32; returns uint16 bits.
+
+    Used only to present the oracle's fp64 dlogits in the library's output type.
+    """
+    f = np.asarray(x, dtype=np.float64).astype(np.float32)
+    u = f.view(np.uint32).astype(np.uint64)
+    nan = np.isnan(f)
+    rounding = ((u >> np.uint64(16)) & np.uint64(1)) + np.uint64(0x7FFF)
+    out = ((u + rounding) >> np.uint64(16)).astype(np.uint16)
+    out[nan] = np.uint16(0x7FC0)
+    return out
+
+
+def log_softmax_rows(z, ids, inv_temp=1.0):
+    """lse_k = log sum_v exp(inv_temp * z_kv);  logp_k = inv_temp * z_k[y_k] - lse_k.
+
+    z is float64 [rows, V]; the max is subtracted before exp (same value, no
+    overflow).  Returns (lse, logp).
+    """
+    x = np.asarray(z, dtype=np.float64) * inv_temp
+    m = x.max(axis=1)
+    s = np.exp(x - m[:, None]).sum(axis=1)
+    lse = m + np.log(s)
+    ids = np.asarray(ids, dtype=np.int64)
+    logp = x[np.arange(x.shape[0]), ids] - lse
+    return lse, logp
+
+
+# ---------------------------------------------------------------------------
+# Eq. 3: the clipped-ratio surrogate L_surr (KL skipped, Fig. 2 caption) and
+# its gradient with respect to the logits.
+# ---------------------------------------------------------------------------
+def grpo_loss_rows(z, ids, old_logp, adv, w, eps_low=0.2, eps_high=0.2, inv_temp=1.0,
+                   grad_scale=1.0, want_dlogits=True):
+    """Clipped surrogate per token and its dlogits, for float64 logits z [rows, V].
+
+    Reading of L_surr (standard PPO/GRPO clip, no dual clip):
+      rho_k   = exp(logp_k - old_k)
+      ell_k   = -min(rho_k * A_k, clip(rho_k, 1 - eps_low, 1 + eps_high) * A_k)
+      loss    = sum_k w_k * ell_k
+    Gradient: d(w_k ell_k)/d logp_k = -w_k A_k rho_k where the unclipped term is
+    the active one (A >= 0 and rho <= 1 + eps_high, or A < 0 and rho >= 1 - eps_low;
+    the closed interval counts as unclipped), else 0; then
+      dlogits_kv = grad_scale * g_k * inv_temp * (1[v = y_k] - softmax_v).
+    Rows with w_k == 0 or an id outside [0, V) are masked: every output is 0.
+    Returns dict(logp, lse, ell, g, rho, active, loss, dlogits, bad_id).
+    """
+    z = np.asarray(z, dtype=np.float64)
+    rows, V = z.shape
+    ids = np.asarray(ids, dtype=np.int64)
+    old_logp = np.asarray(old_logp, dtype=np.float64)
+    adv = np.asarray(adv, dtype=np.float64)
+    w = np.asarray(w, dtype=np.float64)
+
+    bad_id = (w != 0) & ((ids < 0) | (ids >= V))
+    live = (w != 0) & ~bad_id
+    safe_ids = np.where(live, ids, 0)
+
+    lse = np.zeros(rows)
+    logp = np.zeros(rows)
+    if live.any():
+        l_lse, l_logp = log_softmax_rows(z[live], safe_ids[live], inv_temp)
+        lse[live], logp[live] = l_lse, l_logp
+
+    rho = np.where(live, np.exp(logp - old_logp), 0.0)
+    clipped = np.clip(rho, 1.0 - eps_low, 1.0 + eps_high)
+    ell = np.where(live, -np.minimum(rho * adv, clipped * adv), 0.0)
+    active = live & (((adv >= 0) & (rho <= 1.0 + eps_high)) | ((adv < 0) & (rho >= 1.0 - eps_low)))
+    g = np.where(active, -w * adv * rho, 0.0)
+    loss = 0.0
+    for k in range(rows):                      # plain sequential sum
+        loss += w[k] * ell[k]
+
+    dlogits = None
+    if want_dlogits:
+        dlogits = np.zeros((rows, V))
+        for k in np.nonzero(live)[0]:
+            p = np.exp(z[k] * inv_temp - lse[k])
+            onehot = np.zeros(V)
+            onehot[safe_ids[k]] = 1.0
+            dlogits[k] = grad_scale * g[k] * inv_temp * (onehot - p)
+    return dict(logp=logp, lse=lse, ell=ell, g=g, rho=rho, active=active, live=live,
+                loss=loss, dlogits=dlogits, bad_id=bad_id)
+
+
+# ---------------------------------------------------------------------------
+# Fused lm-head variant: logits = hidden . W^T, never stored by the library.
+# ---------------------------------------------------------------------------
+def lmhead_loss_rows(hidden, W, ids, old_logp, adv, w, eps_low=0.2, eps_high=0.2,
+                     inv_temp=1.0, grad_scale=1.0, want_dhidden=True):
+    """The same surrogate on logits z = hidden W^T (fp64), plus dhidden = dlogits . W.
+
+    hidden float64 [rows, H], W float64 [V, H].  Returns the grpo_loss_rows dict
+    with 'dhidden' [rows, H] added.
+    """
+    hidden = np.asarray(hidden, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    z = hidden @ W.T
+    out = grpo_loss_rows(z, ids, old_logp, adv, w, eps_low, eps_high, inv_temp,
+                         grad_scale, want_dlogits=want_dhidden)
+    if want_dhidden:
+        out["dhidden"] = out["dlogits"] @ W
+    return out
