@@ -1,0 +1,360 @@
+#!/usr/bin/env python
+"""Throughput of one LEAP loss hot-path pass (rank advantages -> per-token
+advantages -> clipped GRPO surrogate fwd + fused dlogits) on the single-turn
+GRPO workload: 16 prompts x G = 8 rollouts x 256 token slots (32,768 rows),
+response lengths U{64..256} (the rest is masked padding), vocabulary 151,936,
+bf16 logits ~ N(0, 3^2) with 1% of entries raised by 15, synthetic and seeded.
+
+Prints ONE JSON line (rank 0).  `value` counts valid (response) tokens per
+second over all ranks.  Usage:
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl leap|reference]
+Under torchrun each rank runs its own batch (weak scaling); the only exchange
+is an all-reduce of the two loss normalisers per step.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "rollout tokens/sec through GRPO loss fwd+bwd (V=151936); % of HBM roofline"
+UNIT = "tokens/s"
+V = 151936
+WORKLOAD = ("single-turn GRPO: 16 prompts x G=8 x 256 token slots = 32,768 rows (response lengths U{64..256}, "
+            "rest masked padding), V=151936, bf16 logits N(0,3^2) + 1% spikes of +15, old log-probs = current "
+            "+ N(0,0.05^2), clip eps 0.2/0.2, seq-mean-token-mean aggregation")
+
+# dram bytes (read + write) of one fused_loss_kernel launch on this workload, from an ncu capture of the
+# kernel built from the source file with this SHA-256; reported as null once the source changes.
+KNOWN_TRAFFIC = None
+
+
+def _src_sha():
+    p = os.path.join(ROOT, "paper_2608_01804_gb300", "csrc", "logprob_loss.cu")
+    return hashlib.sha256(open(p, "rb").read()).hexdigest()
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["leap", "reference"], default="leap")
+    ap.add_argument("--e2e-steps", type=int, default=8)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of this GPU's clocks and throttle reasons every 200 ms."""
+
+    FIELDS = ("uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device):
+        try:
+            self.uuid = str(torch.cuda.get_device_properties(device).uuid)
+        except Exception:
+            self.uuid = None
+        self.proc = None
+
+    def start(self):
+        self.out = tempfile.NamedTemporaryFile(mode="w+", suffix=".csv", delete=False)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "--query-gpu=" + self.FIELDS,
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.out, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        self.proc.wait()
+        self.out.flush()
+        self.out.seek(0)
+        sm, smax, power, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.out.read().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            if self.uuid and self.uuid not in f[0] and f[0] not in self.uuid:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+                power.append(float(f[3]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        os.unlink(self.out.name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "samples": len(sm),
+                "power_w_max": max(power), "reasons": sorted(reasons)}
+
+
+def torch_logp(logits, ids, chunk=2048):
+    """Current-policy log-probs with torch's fp32 log_softmax: input generation of
+    the old log-probs only (outside every timed region)."""
+    out = torch.empty(logits.shape[0], dtype=torch.float32, device=logits.device)
+    for a in range(0, logits.shape[0], chunk):
+        b = min(logits.shape[0], a + chunk)
+        out[a:b] = torch.log_softmax(logits[a:b].float(), dim=1).gather(1, ids[a:b].long().view(-1, 1)).view(-1)
+    return out
+
+
+def make_inputs(rank, device):
+    from paper_2608_01804_gb300 import synth
+    batch = synth.single_turn_batch(seed=1 + 1000 * rank)
+    N = batch.N
+    logits = synth.logits(N, V, 3.0, 200 + rank, device, spike_frac=0.01)
+    ids = synth.token_ids(N, V, 201 + rank, device)
+    old = torch_logp(logits, ids) + synth.normal(N, 0.05, 202 + rank, device)
+    return batch, logits, ids, old
+
+
+def valid_tokens(batch):
+    return int(sum(int(batch.seg_offsets[s + 1] - batch.seg_offsets[s])
+                   for s in range(len(batch.seg_rollout)) if batch.seg_turn[s] >= 0))
+
+
+def cpu_oracle_rate(batch, logits, ids, old, seconds, block=32):
+    """The oracle as it stands on a bounded sample of the same workload: the
+    rank/token steps on the whole batch, then the loss fwd + dlogits over rows
+    in order until `seconds` of CPU time; returns (valid tokens/s, rows, valid)."""
+    from oracle import leap_oracle as O
+    G, M = batch.G, batch.M
+    t_total = 0.0
+    t0 = time.perf_counter()
+    orc = O.rank_advantages(batch.pass_turn.reshape(-1, G), batch.num_turns.reshape(-1, G), M, 0, G, 1.0)
+    ta, te = orc["turn_adv"].reshape(-1), orc["T_eff"].reshape(-1)
+    Lc, nv, rv = O.rollout_token_counts(batch.seg_offsets, batch.seg_rollout, batch.seg_turn, te)
+    adv, w = O.token_advantages(batch.N, batch.seg_offsets, batch.seg_rollout, batch.seg_turn, ta, te, M, 0, Lc, nv, rv)
+    t_total += time.perf_counter() - t0
+    rows = valid = 0
+    ids_h = ids.cpu().numpy().astype(np.int64)
+    old_h = old.cpu().numpy().astype(np.float64)
+    while t_total < seconds and rows < batch.N:
+        a, b = rows, min(batch.N, rows + block)
+        bits = logits[a:b].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+        z = O.bf16_bits_to_f64(bits)
+        t0 = time.perf_counter()
+        O.grpo_loss_rows(z, ids_h[a:b], old_h[a:b], adv[a:b], w[a:b])
+        t_total += time.perf_counter() - t0
+        valid += int(np.count_nonzero(w[a:b]))
+        rows = b
+    return valid / t_total, rows, valid, t_total
+
+
+def reference_arm(args):
+    """The oracle (fp64 CPU) as the reference implementation, timed per step on
+    a bounded sample of the same workload; rank 0 only."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from oracle import leap_oracle as O
+    from paper_2608_01804_gb300 import synth
+    batch = synth.single_turn_batch(seed=1)
+    G, M = batch.G, batch.M
+    sample = 48                                   # rows of the loss per step
+    z_bits = synth.logits(sample * 4, V, 3.0, 200, "cpu", spike_frac=0.01)
+    ids = synth.token_ids(sample * 4, V, 201, "cpu")
+    old = torch_logp(z_bits, ids) + synth.normal(sample * 4, 0.05, 202, "cpu")
+    z = O.bf16_bits_to_f64(z_bits.view(torch.int16).numpy().view(np.uint16))
+    ids_h, old_h = ids.numpy().astype(np.int64), old.numpy().astype(np.float64)
+
+    def one_step(k):
+        orc = O.rank_advantages(batch.pass_turn.reshape(-1, G), batch.num_turns.reshape(-1, G), M, 0, G, 1.0)
+        ta, te = orc["turn_adv"].reshape(-1), orc["T_eff"].reshape(-1)
+        Lc, nv, rv = O.rollout_token_counts(batch.seg_offsets, batch.seg_rollout, batch.seg_turn, te)
+        adv, w = O.token_advantages(batch.N, batch.seg_offsets, batch.seg_rollout, batch.seg_turn, ta, te, M, 0,
+                                    Lc, nv, rv)
+        a = (k % 4) * sample
+        live = np.nonzero(w)[0][a:a + sample]
+        O.grpo_loss_rows(z[a:a + sample], ids_h[a:a + sample], old_h[a:a + sample], adv[live], w[live])
+        return len(live)
+
+    for k in range(args.warmup):
+        one_step(k)
+    t0 = time.perf_counter()
+    toks = sum(one_step(k) for k in range(args.steps))
+    dt = time.perf_counter() - t0
+    value = toks / dt
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": WORKLOAD, "sample_rows_per_step": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": "per step: rank/token oracle on the whole batch + loss fwd and dlogits on "
+                                       "%d valid rows" % sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        reference_arm(args)
+        return
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    pg = None
+    if world > 1:
+        torch.distributed.init_process_group("nccl", device_id=device)
+        pg = torch.distributed.group.WORLD
+
+    from paper_2608_01804_gb300 import build
+    build.build()
+    from paper_2608_01804_gb300.step import GrpoStep
+
+    batch, logits, ids, old = make_inputs(rank, device)
+    N = batch.N
+    n_valid = valid_tokens(batch)
+    step = GrpoStep(batch, V, device, gamma=1.0, tau=(0, batch.G), use_gate_in=False)
+    dlogits = torch.empty_like(logits)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if pg is not None:
+            torch.distributed.barrier()
+
+    for _ in range(max(3, args.warmup)):
+        step.run(logits, ids, old, dlogits, pg)
+    torch.cuda.synchronize()
+    live_rows = int((step.w != 0).sum().item())
+    assert live_rows == n_valid
+
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    clocks = ClockSampler(device)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_stop = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for k in range(K):
+        step.advantages(pg)
+        ev[k][0].record(stream)
+        step.loss_pass(logits, ids, old, dlogits)
+        ev[k][1].record(stream)
+    t_stop.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    elapsed_ms = t_start.elapsed_time(t_stop)
+    loss_ms = sum(a.elapsed_time(b) for a, b in ev) / K
+    if pg is not None:
+        t = torch.tensor([elapsed_ms], device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    ms_per_step = elapsed_ms / K
+    value = n_valid * world / (ms_per_step / 1e3)
+
+    peak, peak_kind = measured_peaks()
+    alg_bytes = live_rows * 4 * V + (N - live_rows) * 2 * V + 16 * N
+    achieved = alg_bytes / (loss_ms / 1e3) / 1e9
+    traffic = None
+    if KNOWN_TRAFFIC and KNOWN_TRAFFIC.get("src_sha256") == _src_sha():
+        traffic = KNOWN_TRAFFIC["bytes_per_launch"]
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": traffic, "kernel": "fused_loss_kernel<8,256,10> (+2 reduce launches in the timing)",
+                "algorithmic_bytes_per_launch": alg_bytes, "launch_ms": loss_ms, "peak_source": peak_kind}
+
+    # End to end through the same public calls, inputs copied from pinned host memory every step.
+    e2e = None
+    if not args.no_e2e:
+        host = {k: t.cpu().pin_memory() for k, t in dict(logits=logits, ids=ids, old=old,
+                                                         pass_turn=step.pass_turn, num_turns=step.num_turns,
+                                                         seg_offsets=step.seg_offsets, seg_rollout=step.seg_rollout,
+                                                         seg_turn=step.seg_turn).items()}
+        dev = dict(logits=logits, ids=ids, old=old, pass_turn=step.pass_turn, num_turns=step.num_turns,
+                   seg_offsets=step.seg_offsets, seg_rollout=step.seg_rollout, seg_turn=step.seg_turn)
+        h2d = sum(t.numel() * t.element_size() for t in host.values())
+        loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
+        E = max(1, args.e2e_steps)
+
+        def e2e_step():
+            for k, t in host.items():
+                dev[k].copy_(t, non_blocking=True)
+            step.run(dev["logits"], dev["ids"], dev["old"], dlogits, pg)
+            loss_host.copy_(step.loss, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(E):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        e_ms = a.elapsed_time(b) / E
+        if pg is not None:
+            t = torch.tensor([e_ms], device=device)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            e_ms = float(t.item())
+        e2e = {"value": n_valid * world / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": 4, "ms_per_step": e_ms, "steps": E}
+        del host
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rate, rows, valid, secs = cpu_oracle_rate(batch, logits, ids, old, args.cpu_seconds)
+        cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": "rank/token oracle on the whole batch + loss fwd and dlogits on the first %d rows "
+                         "(%d valid tokens), %.1f s of CPU time" % (rows, valid, secs)}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
+                "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "f32", "data": "synthetic",
+                "config": {"workload": WORKLOAD, "rows_per_step_per_gpu": N, "valid_tokens_per_step_per_gpu": n_valid,
+                           "vocab": V, "logits_dtype": "bf16", "l2": "inputs larger than L2 (9.96 GB of logits "
+                           "read and 9.96 GB of dlogits written per step)", "parallelism": "dp%d" % world},
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+                "gpu_launches": K * GrpoStep.LAUNCHES_PER_RUN, "clocks": clk}
+        print(json.dumps(line), flush=True)
+    if pg is not None:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

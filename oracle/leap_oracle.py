@@ -53,38 +53,20 @@ def tiers_and_gate(pass_turn, num_turns, M, tau_min, tau_max, gate_in=None):
     """
     pass_turn = np.asarray(pass_turn, dtype=np.int64)
     num_turns = np.asarray(num_turns, dtype=np.int64)
-    num_groups, G = pass_turn.shape
+    m, T = pass_turn, num_turns
 
-    bad = np.zeros((num_groups, G), dtype=bool)
-    n_fail = np.zeros(num_groups, dtype=np.int64)
-    gate = np.zeros(num_groups, dtype=np.uint8)
-    r = np.zeros((num_groups, G), dtype=np.int64)
-    T_eff = np.zeros((num_groups, G), dtype=np.int64)
-
-    for g in range(num_groups):
-        for i in range(G):
-            m, T = pass_turn[g, i], num_turns[g, i]
-            if m < 0 or m > M or T < 1 or T > M or (m >= 1 and m > T):
-                bad[g, i] = True
-        # Eq. 1 over first-turn outcomes (a malformed rollout counts as failed).
-        for i in range(G):
-            if bad[g, i] or pass_turn[g, i] != 1:
-                n_fail[g] += 1
-        if gate_in is not None:
-            gate[g] = 1 if gate_in[g] != 0 else 0
-        else:
-            gate[g] = 1 if (tau_min <= n_fail[g] <= tau_max) else 0   # Eq. 2
-        for i in range(G):
-            if bad[g, i]:
-                r[g, i], T_eff[g, i] = 0, 0
-                continue
-            m = pass_turn[g, i]
-            if gate[g] == 0:
-                r[g, i] = M if m == 1 else 0
-                T_eff[g, i] = 1
-            else:
-                r[g, i] = (M - m + 1) if m >= 1 else 0
-                T_eff[g, i] = num_turns[g, i]
+    bad = (m < 0) | (m > M) | (T < 1) | (T > M) | ((m >= 1) & (m > T))
+    # Eq. 1 over first-turn outcomes (a malformed rollout counts as failed).
+    n_fail = np.sum(bad | (m != 1), axis=1).astype(np.int64)
+    if gate_in is not None:
+        gate = (np.asarray(gate_in) != 0).astype(np.uint8)
+    else:
+        gate = ((tau_min <= n_fail) & (n_fail <= tau_max)).astype(np.uint8)    # Eq. 2
+    on = gate[:, None] == 1
+    r_on = np.where(m >= 1, M - m + 1, 0)          # tier rule, expanded group
+    r_off = np.where(m == 1, M, 0)                 # truncated to turn 1
+    r = np.where(bad, 0, np.where(on, r_on, r_off)).astype(np.int64)
+    T_eff = np.where(bad, 0, np.where(on, T, 1)).astype(np.int64)
     return n_fail, gate, r, T_eff, bad
 
 
@@ -143,13 +125,11 @@ def turn_advantages(A, T_eff, gamma, M):
     """
     A = np.asarray(A, dtype=np.float64)
     T_eff = np.asarray(T_eff, dtype=np.int64)
-    num_groups, G = A.shape
-    out = np.zeros((num_groups, G, M), dtype=np.float64)
-    for g in range(num_groups):
-        for i in range(G):
-            beta = gamma if A[g, i] >= 0 else 1.0
-            for t in range(T_eff[g, i]):
-                out[g, i, t] = (beta ** (T_eff[g, i] - t - 1)) * A[g, i]
+    beta = np.where(A >= 0, gamma, 1.0)
+    out = np.zeros(A.shape + (M,), dtype=np.float64)
+    for t in range(M):
+        exponent = T_eff - t - 1
+        out[..., t] = np.where(t < T_eff, beta ** np.maximum(exponent, 0) * A, 0.0)
     return out
 
 

@@ -1,0 +1,570 @@
+// Token log-probs, the clipped GRPO surrogate (Eq. 3, KL skipped) with its
+// deterministic masked reduction, and the dlogits backward.
+//
+// Kernels
+//   row_stream_kernel  one pass over each logits row with an online
+//                      (max, sum) -> log-probs, or the loss forward without
+//                      dlogits.  2V bytes read per row.
+//   fused_loss_kernel  forward + backward in one pass.  A row is split over a
+//                      cluster of C CTAs; each CTA keeps its slice in
+//                      registers, the CTAs exchange one (max, sum) pair
+//                      through distributed shared memory, then each writes
+//                      its dlogits slice.  2V read + 2V written per row.
+//   split_bwd_kernel   dlogits from a saved lse: 2V read + 2V written.
+//   reduce kernels     fixed-order fp64 sum of the per-row loss terms.
+#include "../../include/leap.h"
+#include "leap_common.cuh"
+#include "leap_internal.h"
+
+#include <algorithm>
+#include <math.h>
+#include <mutex>
+
+namespace leap {
+namespace {
+
+__device__ __forceinline__ uint4 neg_inf4() {
+    return make_uint4(kNegInfBf16x2, kNegInfBf16x2, kNegInfBf16x2, kNegInfBf16x2);
+}
+
+// Sets elements n..7 of an 8 x bf16 vector to -inf (row tail beyond V).
+__device__ __forceinline__ void mask_tail(uint4& x, int n) {
+    uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        if (j >= n) {
+            if (j & 1) w[j >> 1] = (w[j >> 1] & 0x0000ffffu) | 0xff800000u;
+            else       w[j >> 1] = (w[j >> 1] & 0xffff0000u) | 0x0000ff80u;
+        }
+    }
+    x = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+__device__ __forceinline__ uint32_t max8(const uint4& x, uint32_t m) {
+    return max_bf16x2(max_bf16x2(m, x.x), max_bf16x2(max_bf16x2(x.y, x.z), x.w));
+}
+
+// Stores vector vi of a dlogits row; the row's last vector keeps columns >= V intact.
+__device__ __forceinline__ void store_vec(uint4* drow, int64_t vi, uint4 val, int64_t V8, int tailn) {
+    if (tailn == 0 || vi != V8 - 1) {
+        st_stream(drow + vi, val);
+    } else {
+        uint16_t* p = reinterpret_cast<uint16_t*>(drow + vi);
+        const uint32_t w[4] = {val.x, val.y, val.z, val.w};
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+            if (j < tailn) p[j] = (uint16_t)((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xffffu));
+    }
+}
+
+__device__ __forceinline__ float bf16_at(const uint16_t* p) {
+    return __uint_as_float(((uint32_t)*p) << 16);
+}
+
+// sum over the 8 elements of 2^(z * c1 - mc)
+__device__ __forceinline__ float exp_sum8(const uint4& x, float c1, float mc) {
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        a0 += ex2(fmaf(bf16_lo(w[q]), c1, -mc));
+        a1 += ex2(fmaf(bf16_hi(w[q]), c1, -mc));
+    }
+    return a0 + a1;
+}
+
+// dlogits of one vector: coef * (1[v = y] - 2^(z c1 - K)); `yl` is the target's
+// lane in this vector or -1.
+__device__ __forceinline__ uint4 dlogit8(const uint4& x, float c1, float K, float coef, int yl) {
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        float lo = -coef * ex2(fmaf(bf16_lo(w[q]), c1, -K));
+        float hi = -coef * ex2(fmaf(bf16_hi(w[q]), c1, -K));
+        if (yl == 2 * q) lo += coef;
+        if (yl == 2 * q + 1) hi += coef;
+        o[q] = pack_bf16x2(lo, hi);
+    }
+    return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+struct TokenLoss {
+    float logp, lse, ell, rho, g;
+    bool active;
+};
+
+// Clipped surrogate for one token given its row max m (raw logits), the
+// scaled sum s = sum_v 2^((z_v - m) inv_temp log2 e) and the target logit zy.
+__device__ __forceinline__ TokenLoss token_loss(const RowArgs& a, float m, float s, float zy, float old,
+                                                float A, float wk) {
+    TokenLoss r;
+    const float lnS = logf(s);
+    r.lse = fmaf(m, a.inv_temp, lnS);
+    r.logp = a.inv_temp * (zy - m) - lnS;
+    r.rho = expf(r.logp - old);
+    const float lo = 1.f - a.eps_low, hi = 1.f + a.eps_high;
+    const float clipped = fminf(fmaxf(r.rho, lo), hi);
+    r.ell = -fminf(r.rho * A, clipped * A);
+    r.active = (A >= 0.f) ? (r.rho <= hi) : (r.rho >= lo);
+    r.g = r.active ? -wk * A * r.rho : 0.f;
+    return r;
+}
+
+__device__ __forceinline__ void write_row_outputs(const RowArgs& a, int64_t row, const TokenLoss& r, float wk) {
+    if (a.logp) a.logp[row] = r.logp;
+    if (a.lse) a.lse[row] = r.lse;
+    if (a.ell) a.ell[row] = r.ell;
+    if (a.ws_contrib) {
+        a.ws_contrib[row] = (double)wk * (double)r.ell;
+        a.ws_rho[row] = r.rho;
+        a.ws_flag[row] = (uint8_t)(1u | (r.active ? 0u : 2u));
+    }
+}
+
+__device__ __forceinline__ void write_masked_outputs(const RowArgs& a, int64_t row) {
+    if (a.logp) a.logp[row] = 0.f;
+    if (a.lse) a.lse[row] = 0.f;
+    if (a.ell) a.ell[row] = 0.f;
+    if (a.ws_contrib) {
+        a.ws_contrib[row] = 0.0;
+        a.ws_rho[row] = 0.f;
+        a.ws_flag[row] = 0;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Streaming single pass.  TPR threads per row (32: several rows per CTA;
+// 512: one row per CTA), U vectors of 8 bf16 in flight per thread.
+// mode 0: log-probs (every row read); mode 1: loss forward (w == 0 rows skipped).
+// ---------------------------------------------------------------------------
+template <int TPR, int U>
+__global__ void __launch_bounds__(512) row_stream_kernel(RowArgs a, int mode) {
+    __shared__ float2 wpart[16];
+    const int t = threadIdx.x % TPR;
+    const int64_t row = (int64_t)blockIdx.x * (blockDim.x / TPR) + threadIdx.x / TPR;
+    if (row >= a.N) return;  // uniform per row group (one row per CTA when TPR = 512)
+    const int V = a.V;
+    const float wk = (mode == 1) ? a.w[row] : 1.f;
+    const int id = a.ids[row];
+    const bool bad = (wk != 0.f) && (id < 0 || id >= V);
+    if (mode == 1 && (wk == 0.f || bad)) {
+        if (t == 0) {
+            write_masked_outputs(a, row);
+            if (bad) flag_status(a.status, LEAP_DEV_BAD_ID);
+        }
+        return;
+    }
+    const uint16_t* zr = a.logits + row * a.ld;
+    float zy = 0.f;
+    if (t == 0 && !bad) zy = bf16_at(zr + id);
+
+    const uint4* zrow = reinterpret_cast<const uint4*>(zr);
+    const int64_t V8 = ((int64_t)V + 7) >> 3;
+    const int tailn = V & 7;
+    const float c1 = a.inv_temp * kLog2e;
+    float m = -INFINITY, s = 0.f;
+    for (int64_t v0 = t; v0 < V8; v0 += (int64_t)TPR * U) {
+        uint4 x[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t vi = v0 + (int64_t)u * TPR;
+            x[u] = (vi < V8) ? ld_stream(zrow + vi) : neg_inf4();
+            if (tailn && vi == V8 - 1) mask_tail(x[u], tailn);
+        }
+        uint32_t mx = kNegInfBf16x2;
+#pragma unroll
+        for (int u = 0; u < U; ++u) mx = max8(x[u], mx);
+        const float bm = fmaxf(bf16_lo(mx), bf16_hi(mx));
+        if (bm == -INFINITY) continue;
+        const float mn = fmaxf(m, bm);
+        const float mc = mn * c1;
+        float acc = 0.f;
+#pragma unroll
+        for (int u = 0; u < U; ++u) acc += exp_sum8(x[u], c1, mc);
+        s = (s == 0.f) ? acc : fmaf(s, ex2((m - mn) * c1), acc);
+        m = mn;
+    }
+    warp_lse_merge(m, s, c1);
+    if (TPR > 32) {
+        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+        if (lane == 0) wpart[warp] = make_float2(m, s);
+        __syncthreads();
+        if (warp == 0) {
+            const float2 p = (lane < TPR / 32) ? wpart[lane] : make_float2(-INFINITY, 0.f);
+            m = p.x;
+            s = p.y;
+            warp_lse_merge(m, s, c1);
+        }
+    }
+    if (t != 0) return;
+    if (mode == 0) {
+        const float lnS = logf(s);
+        if (a.lse) a.lse[row] = fmaf(m, a.inv_temp, lnS);
+        if (bad) {
+            a.logp[row] = 0.f;
+            flag_status(a.status, LEAP_DEV_BAD_ID);
+        } else {
+            a.logp[row] = a.inv_temp * (zy - m) - lnS;
+        }
+        return;
+    }
+    const TokenLoss r = token_loss(a, m, s, zy, a.old_logp[row], a.adv[row], wk);
+    write_row_outputs(a, row, r, wk);
+}
+
+// ---------------------------------------------------------------------------
+// Fused forward + backward.  Grid = N * C CTAs; the C consecutive CTAs of a
+// cluster share one row.  CTA c owns 16-byte vectors [c * per, (c+1) * per)
+// of the row (per = ceil(V8 / C) <= T * NV) and holds them in registers
+// between the forward reduction and the dlogits write.
+// ---------------------------------------------------------------------------
+template <int C, int T, int NV>
+__global__ void __launch_bounds__(T) fused_loss_kernel(RowArgs a) {
+    __shared__ float2 wpart[T / 32];
+    __shared__ float2 cta_part;  // read by the other CTAs of the cluster
+    __shared__ float bc[2];
+    const uint32_t crank = (C > 1) ? cluster_ctarank() : 0u;
+    const int64_t row = blockIdx.x / C;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int V = a.V;
+    const int64_t V8 = ((int64_t)V + 7) >> 3;
+    const int64_t per = (V8 + C - 1) / C;
+    const int64_t vbeg = (int64_t)crank * per;
+    const int64_t vend = min(vbeg + per, V8);
+    const int tailn = V & 7;
+    const float wk = a.w[row];
+    const int id = a.ids[row];
+    const bool bad = (wk != 0.f) && (id < 0 || id >= V);
+    uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
+
+    if (wk == 0.f || bad) {  // masked row: the same branch for the whole cluster
+#pragma unroll
+        for (int k = 0; k < NV; ++k) {
+            const int64_t vi = vbeg + t + (int64_t)k * T;
+            if (vi < vend) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
+        }
+        if (crank == 0 && t == 0) {
+            write_masked_outputs(a, row);
+            if (bad) flag_status(a.status, LEAP_DEV_BAD_ID);
+        }
+        return;
+    }
+
+    const uint16_t* zr = a.logits + row * a.ld;
+    float zy = 0.f;
+    if (t == 0) zy = bf16_at(zr + id);
+    const uint4* zrow = reinterpret_cast<const uint4*>(zr);
+    uint4 x[NV];
+#pragma unroll
+    for (int k = 0; k < NV; ++k) {
+        const int64_t vi = vbeg + t + (int64_t)k * T;
+        x[k] = (vi < vend) ? ld_stream(zrow + vi) : neg_inf4();
+        if (tailn && vi == V8 - 1) mask_tail(x[k], tailn);
+    }
+    uint32_t mx = kNegInfBf16x2;
+#pragma unroll
+    for (int k = 0; k < NV; ++k) mx = max8(x[k], mx);
+    float m = fmaxf(bf16_lo(mx), bf16_hi(mx));
+    const float c1 = a.inv_temp * kLog2e;
+    float s = 0.f;
+    if (m != -INFINITY) {
+        const float mc = m * c1;
+        float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+        for (int k = 0; k < NV; k += 2) {
+            s0 += exp_sum8(x[k], c1, mc);
+            if (k + 1 < NV) s1 += exp_sum8(x[k + 1], c1, mc);
+        }
+        s = s0 + s1;
+    }
+    warp_lse_merge(m, s, c1);
+    if (lane == 0) wpart[warp] = make_float2(m, s);
+    __syncthreads();
+    if (warp == 0) {
+        const float2 p = (lane < T / 32) ? wpart[lane] : make_float2(-INFINITY, 0.f);
+        m = p.x;
+        s = p.y;
+        warp_lse_merge(m, s, c1);
+        if (lane == 0) cta_part = make_float2(m, s);
+    }
+    if (C > 1) {
+        cluster_arrive_release();
+        cluster_wait_acquire();  // every CTA's cta_part is visible
+        if (warp == 0) {
+            const float2 p = (lane < C) ? ld_cluster_f32x2(cluster_map(smem_addr(&cta_part), (uint32_t)lane))
+                                        : make_float2(-INFINITY, 0.f);
+            m = p.x;
+            s = p.y;
+            warp_lse_merge(m, s, c1);
+        }
+        cluster_arrive_release();  // this CTA is done reading its peers' shared memory
+    }
+    if (t == 0) {
+        const TokenLoss r = token_loss(a, m, s, zy, a.old_logp[row], a.adv[row], wk);
+        bc[0] = fmaf(m, c1, log2f(s));               // log2 of the softmax denominator
+        bc[1] = a.grad_scale * r.g * a.inv_temp;      // dlogits scale
+        if (crank == 0) write_row_outputs(a, row, r, wk);
+    }
+    __syncthreads();
+    const float K = bc[0], coef = bc[1];
+    const int64_t yv = id >> 3;
+    const int ylane = id & 7;
+#pragma unroll
+    for (int k = 0; k < NV; ++k) {
+        const int64_t vi = vbeg + t + (int64_t)k * T;
+        if (vi < vend) {
+            const uint4 d = (coef == 0.f) ? make_uint4(0, 0, 0, 0)
+                                          : dlogit8(x[k], c1, K, coef, vi == yv ? ylane : -1);
+            store_vec(drow, vi, d, V8, tailn);
+        }
+    }
+    if (C > 1) cluster_wait_acquire();  // peers finished reading cta_part
+}
+
+// ---------------------------------------------------------------------------
+// Split backward from the saved lse.  Every thread recomputes the row's scalar
+// coefficient from broadcast loads, so no block synchronisation is needed.
+// ---------------------------------------------------------------------------
+template <int TPR, int U>
+__global__ void __launch_bounds__(512) split_bwd_kernel(RowArgs a) {
+    const int t = threadIdx.x % TPR;
+    const int64_t row = (int64_t)blockIdx.x * (blockDim.x / TPR) + threadIdx.x / TPR;
+    if (row >= a.N) return;
+    const int V = a.V;
+    const int64_t V8 = ((int64_t)V + 7) >> 3;
+    const int tailn = V & 7;
+    const float wk = a.w[row];
+    const int id = a.ids[row];
+    const bool bad = (wk != 0.f) && (id < 0 || id >= V);
+    uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
+    float coef = 0.f, K = 0.f;
+    if (wk != 0.f && !bad) {
+        const float lse = a.lse_in[row];
+        const float logp = a.inv_temp * bf16_at(a.logits + row * a.ld + id) - lse;
+        const float A = a.adv[row];
+        const float rho = expf(logp - a.old_logp[row]);
+        const bool active = (A >= 0.f) ? (rho <= 1.f + a.eps_high) : (rho >= 1.f - a.eps_low);
+        coef = active ? a.grad_scale * (-wk * A * rho) * a.inv_temp : 0.f;
+        K = lse * kLog2e;
+    }
+    if (bad && t == 0) flag_status(a.status, LEAP_DEV_BAD_ID);
+    const uint4* zrow = reinterpret_cast<const uint4*>(a.logits + row * a.ld);
+    const float c1 = a.inv_temp * kLog2e;
+    const int64_t yv = bad ? -1 : (id >> 3);
+    const int ylane = id & 7;
+    for (int64_t v0 = t; v0 < V8; v0 += (int64_t)TPR * U) {
+        if (coef == 0.f) {
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int64_t vi = v0 + (int64_t)u * TPR;
+                if (vi < V8) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
+            }
+            continue;
+        }
+        uint4 x[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t vi = v0 + (int64_t)u * TPR;
+            x[u] = (vi < V8) ? ld_stream(zrow + vi) : neg_inf4();
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t vi = v0 + (int64_t)u * TPR;
+            if (vi < V8) store_vec(drow, vi, dlogit8(x[u], c1, K, coef, vi == yv ? ylane : -1), V8, tailn);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Deterministic reduction: block b sums rows [b R, (b+1) R) in a fixed order,
+// then one block sums the block partials in a fixed order.
+// ---------------------------------------------------------------------------
+constexpr int kRedThreads = 256;
+
+template <typename Tv>
+__device__ __forceinline__ Tv block_sum_fixed(Tv v, Tv* sh) {
+    sh[threadIdx.x] = v;
+    __syncthreads();
+    for (int o = blockDim.x / 2; o > 0; o >>= 1) {
+        if ((int)threadIdx.x < o) sh[threadIdx.x] += sh[threadIdx.x + o];
+        __syncthreads();
+    }
+    const Tv r = sh[0];
+    __syncthreads();
+    return r;
+}
+
+__global__ void __launch_bounds__(kRedThreads) reduce_partial_kernel(LossWorkspace ws, int64_t N) {
+    __shared__ double shd[kRedThreads];
+    __shared__ long long shl[kRedThreads];
+    const int64_t lo = (int64_t)blockIdx.x * kReduceRowsPerBlock;
+    const int64_t hi = min(N, lo + kReduceRowsPerBlock);
+    double l = 0.0, rs = 0.0;
+    long long live = 0, clip = 0;
+    for (int64_t i = lo + threadIdx.x; i < hi; i += kRedThreads) {
+        l += ws.contrib[i];
+        rs += (double)ws.rho[i];
+        const uint8_t f = ws.flag[i];
+        live += (f & 1u);
+        clip += (f >> 1) & 1u;
+    }
+    l = block_sum_fixed(l, shd);
+    rs = block_sum_fixed(rs, shd);
+    live = block_sum_fixed(live, shl);
+    clip = block_sum_fixed(clip, shl);
+    if (threadIdx.x == 0) {
+        ws.part_loss[blockIdx.x] = l;
+        ws.part_rho[blockIdx.x] = rs;
+        ws.part_live[blockIdx.x] = live;
+        ws.part_clip[blockIdx.x] = clip;
+    }
+}
+
+__global__ void __launch_bounds__(kRedThreads) reduce_final_kernel(LossWorkspace ws, float* loss,
+                                                                    leap_loss_stats_t* stats, int accumulate) {
+    __shared__ double shd[kRedThreads];
+    __shared__ long long shl[kRedThreads];
+    double l = 0.0, rs = 0.0;
+    long long live = 0, clip = 0;
+    for (int64_t b = threadIdx.x; b < ws.nblk; b += kRedThreads) {
+        l += ws.part_loss[b];
+        rs += ws.part_rho[b];
+        live += ws.part_live[b];
+        clip += ws.part_clip[b];
+    }
+    l = block_sum_fixed(l, shd);
+    rs = block_sum_fixed(rs, shd);
+    live = block_sum_fixed(live, shl);
+    clip = block_sum_fixed(clip, shl);
+    if (threadIdx.x == 0) {
+        loss[0] = accumulate ? loss[0] + (float)l : (float)l;
+        if (stats) {
+            if (accumulate) {
+                stats->loss_sum += l;
+                stats->rho_sum += rs;
+                stats->live_tokens += live;
+                stats->clipped_tokens += clip;
+            } else {
+                stats->loss_sum = l;
+                stats->rho_sum = rs;
+                stats->live_tokens = live;
+                stats->clipped_tokens = clip;
+            }
+        }
+    }
+}
+
+// ---- fused-kernel configurations ------------------------------------------
+struct FusedCfg {
+    int C, T, NV;
+};
+constexpr FusedCfg kFused[] = {
+    {1, 128, 1}, {1, 256, 4}, {1, 512, 8}, {4, 512, 8}, {8, 256, 10}, {8, 512, 8}, {8, 512, 16},
+};
+
+template <int C, int T, int NV>
+cudaError_t launch_fused_cfg(const RowArgs& a, cudaStream_t s) {
+    auto kern = fused_loss_kernel<C, T, NV>;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(a.N * C), 1, 1);
+    cfg.blockDim = dim3(T, 1, 1);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    if (C > 1) {
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = C;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+    }
+    return cudaLaunchKernelEx(&cfg, kern, a);
+}
+
+}  // namespace
+
+size_t loss_workspace_bytes(int64_t N) {
+    const int64_t nblk = std::max<int64_t>(1, (N + kReduceRowsPerBlock - 1) / kReduceRowsPerBlock);
+    auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
+    return al(N * sizeof(double)) + al(N * sizeof(float)) + al(N) + 4 * al(nblk * 8);
+}
+
+LossWorkspace carve_loss_workspace(void* base, int64_t N) {
+    auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
+    LossWorkspace w;
+    w.nblk = std::max<int64_t>(1, (N + kReduceRowsPerBlock - 1) / kReduceRowsPerBlock);
+    char* p = static_cast<char*>(base);
+    w.contrib = reinterpret_cast<double*>(p);
+    p += al(N * sizeof(double));
+    w.rho = reinterpret_cast<float*>(p);
+    p += al(N * sizeof(float));
+    w.flag = reinterpret_cast<uint8_t*>(p);
+    p += al(N);
+    w.part_loss = reinterpret_cast<double*>(p);
+    p += al(w.nblk * 8);
+    w.part_rho = reinterpret_cast<double*>(p);
+    p += al(w.nblk * 8);
+    w.part_live = reinterpret_cast<long long*>(p);
+    p += al(w.nblk * 8);
+    w.part_clip = reinterpret_cast<long long*>(p);
+    return w;
+}
+
+int64_t fused_max_vocab() {
+    const FusedCfg& c = kFused[sizeof(kFused) / sizeof(kFused[0]) - 1];
+    return (int64_t)c.C * c.T * c.NV * 8;
+}
+
+cudaError_t launch_row_stream(const RowArgs& a, int mode, cudaStream_t s) {
+    if (a.N == 0) return cudaSuccess;
+    const int64_t V8 = ((int64_t)a.V + 7) >> 3;
+    if (V8 <= 128) {
+        const int64_t blocks = (a.N + 7) / 8;
+        row_stream_kernel<32, 4><<<(unsigned)blocks, 256, 0, s>>>(a, mode);
+    } else {
+        row_stream_kernel<512, 8><<<(unsigned)a.N, 512, 0, s>>>(a, mode);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_split_bwd(const RowArgs& a, cudaStream_t s) {
+    if (a.N == 0) return cudaSuccess;
+    const int64_t V8 = ((int64_t)a.V + 7) >> 3;
+    if (V8 <= 128) {
+        const int64_t blocks = (a.N + 7) / 8;
+        split_bwd_kernel<32, 4><<<(unsigned)blocks, 256, 0, s>>>(a);
+    } else {
+        split_bwd_kernel<512, 4><<<(unsigned)a.N, 512, 0, s>>>(a);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fused_loss(const RowArgs& a, cudaStream_t s) {
+    if (a.N == 0) return cudaSuccess;
+    const int64_t V8 = ((int64_t)a.V + 7) >> 3;
+    for (const FusedCfg& c : kFused) {
+        const int64_t per = (V8 + c.C - 1) / c.C;
+        if (per > (int64_t)c.T * c.NV) continue;
+        if (c.C == 1 && c.T == 128) return launch_fused_cfg<1, 128, 1>(a, s);
+        if (c.C == 1 && c.T == 256) return launch_fused_cfg<1, 256, 4>(a, s);
+        if (c.C == 1 && c.T == 512) return launch_fused_cfg<1, 512, 8>(a, s);
+        if (c.C == 4) return launch_fused_cfg<4, 512, 8>(a, s);
+        if (c.C == 8 && c.T == 256) return launch_fused_cfg<8, 256, 10>(a, s);
+        if (c.C == 8 && c.NV == 8) return launch_fused_cfg<8, 512, 8>(a, s);
+        return launch_fused_cfg<8, 512, 16>(a, s);
+    }
+    return cudaErrorNotSupported;
+}
+
+cudaError_t launch_loss_reduce(const LossWorkspace& ws, int64_t N, float* loss, void* stats, bool accumulate,
+                               cudaStream_t s) {
+    // nblk >= 1: with N == 0 the single block writes zero partials.
+    reduce_partial_kernel<<<(unsigned)ws.nblk, kRedThreads, 0, s>>>(ws, N);
+    reduce_final_kernel<<<1, kRedThreads, 0, s>>>(ws, loss, static_cast<leap_loss_stats_t*>(stats),
+                                                  accumulate ? 1 : 0);
+    return cudaGetLastError();
+}
+
+}  // namespace leap

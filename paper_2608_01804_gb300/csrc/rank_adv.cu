@@ -1,0 +1,266 @@
+// Rank-based advantages (Sec. 3.1 Eqs. 1-2, Sec. 3.2 Eqs. 4-6 + GRPO step,
+// Sec. 3.3 discount) and the per-token scatter of the turn advantages.
+//
+// One warp per rollout group.  Lane l owns rollouts l, l + 32, ...  Because
+// the paper's comparator looks only at the tier r in [0, M], the O(G^2)
+// tournament of Eq. 5 collapses to a histogram of r: N_worse = #peers with a
+// lower tier, N_better = #peers with a higher tier.  The histogram is built
+// with warp ballots, so the whole group stays in registers.
+#include "leap_common.cuh"
+#include "leap_internal.h"
+
+#include <math.h>
+
+namespace leap {
+namespace {
+
+constexpr int kMaxM = 8;
+
+template <int J>  // rollouts per lane: G <= 32 * J
+__global__ void __launch_bounds__(256) rank_adv_kernel(RankArgs a) {
+    const int lane = threadIdx.x & 31;
+    const int64_t group = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (group >= a.num_groups) return;
+    const int G = a.G, M = a.M;
+    const int64_t base = group * G;
+
+    int r[J], T[J];
+    bool valid[J], bad[J];
+    int n_fail = 0;
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+        const int i = lane + 32 * j;
+        valid[j] = i < G;
+        int pt = 0, nt = 1;
+        if (valid[j]) {
+            pt = a.pass_turn[base + i];
+            nt = a.num_turns[base + i];
+        }
+        bad[j] = valid[j] && (pt < 0 || pt > M || nt < 1 || nt > M || (pt >= 1 && pt > nt));
+        // Eq. 1 over first-turn outcomes; a malformed outcome counts as failed.
+        const bool fail1 = valid[j] && (bad[j] || pt != 1);
+        n_fail += __popc(__ballot_sync(0xffffffffu, fail1));
+        r[j] = pt;   // temporarily the pass turn
+        T[j] = nt;
+    }
+    // Eq. 2 (or the recorded gate).
+    const bool gate = a.gate_in ? (a.gate_in[group] != 0) : (a.tau_min <= n_fail && n_fail <= a.tau_max);
+
+    // Tier rule of Sec. 3.2; gated-off groups ran turn 1 only.
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+        const int pt = r[j];
+        if (!valid[j] || bad[j]) {
+            r[j] = 0;
+            T[j] = 0;
+        } else if (!gate) {
+            r[j] = (pt == 1) ? M : 0;
+            T[j] = 1;
+        } else {
+            r[j] = (pt >= 1) ? (M - pt + 1) : 0;
+        }
+        if (bad[j]) flag_status(a.status, 2u);
+    }
+
+    // Histogram of tiers 0..M via ballots.
+    int hist[kMaxM + 1];
+#pragma unroll
+    for (int b = 0; b <= kMaxM; ++b) {
+        int c = 0;
+        if (b <= M) {
+#pragma unroll
+            for (int j = 0; j < J; ++j) c += __popc(__ballot_sync(0xffffffffu, valid[j] && r[j] == b));
+        }
+        hist[b] = c;
+    }
+
+    // Eq. 5 from the histogram; Eq. 6; sum of squared net scores (exact).
+    int d[J];
+    long long dd = 0;
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+        int nw = 0, nb = 0;
+#pragma unroll
+        for (int b = 0; b <= kMaxM; ++b) {
+            nw += (b < r[j]) ? hist[b] : 0;
+            nb += (b > r[j]) ? hist[b] : 0;
+        }
+        d[j] = nw - nb;
+        if (valid[j]) {
+            dd += (long long)d[j] * d[j];
+            const int64_t i = base + lane + 32 * j;
+            if (a.n_worse) a.n_worse[i] = nw;
+            if (a.n_better) a.n_better[i] = nb;
+            if (a.r_out) a.r_out[i] = (uint8_t)r[j];
+            a.T_eff[i] = (uint8_t)T[j];
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) dd += __shfl_xor_sync(0xffffffffu, dd, o);
+
+    // GRPO standardisation.  mean_g R = 0 exactly (every strict pair adds +1
+    // and -1 to the net scores), so A_i = d_i / ((G - 1) (std + eps)) with
+    // std = sqrt(sum d^2 / (G - 1)^2 / den), den = G - 1 (unbiased) or G.
+    const float gm1 = (float)(G - 1);
+    float inv_scale;
+    if (a.norm == 1) {
+        inv_scale = 0.f;  // unused
+    } else {
+        const double den = a.std_unbiased ? (double)(G - 1) : (double)G;
+        const double stdv = sqrt((double)dd / ((double)(G - 1) * (double)(G - 1) * den));
+        inv_scale = (float)(1.0 / ((double)(G - 1) * (stdv + (double)a.eps_std)));
+    }
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+        if (!valid[j]) continue;
+        const int64_t i = base + lane + 32 * j;
+        const float Ri = (float)d[j] / gm1;                      // Eq. 6, correctly rounded
+        const float Ai = (a.norm == 1) ? Ri : (float)d[j] * inv_scale;
+        if (a.R) a.R[i] = Ri;
+        if (a.A) a.A[i] = Ai;
+        // Sec. 3.3: beta = gamma for A >= 0, else 1; last turn keeps A.
+        const float beta = (Ai >= 0.f) ? a.gamma : 1.f;
+        float* ta = a.turn_adv + i * M;
+        float p = Ai;
+        for (int t = M - 1; t >= 0; --t) {
+            if (t < T[j]) {
+                ta[t] = p;
+                p *= beta;
+            } else {
+                ta[t] = 0.f;
+            }
+        }
+    }
+    if (lane == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
+}
+
+template <int J>
+cudaError_t launch_rank_j(const RankArgs& a, cudaStream_t s) {
+    const int warps = 8;
+    const int64_t blocks = ((int64_t)a.num_groups + warps - 1) / warps;
+    rank_adv_kernel<J><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+// ---- per-rollout token counts --------------------------------------------
+
+__global__ void zero_counts_kernel(int32_t* L, int32_t n, int64_t* totals) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        L[i] = 0;
+    if (blockIdx.x == 0 && threadIdx.x < 2) totals[threadIdx.x] = 0;
+}
+
+// Validates segment s; returns false (and flags) when it is malformed.
+__device__ __forceinline__ bool segment_ok(const SegArgs& a, int64_t s, int32_t& lo, int32_t& hi,
+                                           int32_t& i, int32_t& t) {
+    lo = a.seg_offsets[s];
+    hi = a.seg_offsets[s + 1];
+    t = a.seg_turn[s];
+    i = a.seg_rollout[s];
+    const bool ok = lo >= 0 && hi >= lo && (int64_t)hi <= a.N && t < a.M &&
+                    (t < 0 || (i >= 0 && i < a.n_rollouts));
+    return ok;
+}
+
+__global__ void segment_count_kernel(SegArgs a) {
+    const int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (s >= a.num_segs) return;
+    int32_t lo, hi, i, t;
+    if (!segment_ok(a, s, lo, hi, i, t)) {
+        flag_status(a.status, 4u);
+        return;
+    }
+    if (t < 0 || hi == lo) return;
+    if (t < (int)a.T_eff[i]) atomicAdd(&a.L_out[i], hi - lo);
+}
+
+__global__ void totals_kernel(const int32_t* L, int32_t n, int64_t* totals) {
+    long long tok = 0, roll = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const int32_t l = L[i];
+        tok += l;
+        roll += (l > 0);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        tok += __shfl_xor_sync(0xffffffffu, tok, o);
+        roll += __shfl_xor_sync(0xffffffffu, roll, o);
+    }
+    __shared__ long long st[2][32];
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) { st[0][w] = tok; st[1][w] = roll; }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        long long a0 = 0, a1 = 0;
+        for (int k = 0; k < (int)(blockDim.x >> 5); ++k) { a0 += st[0][k]; a1 += st[1][k]; }
+        if (a0) atomicAdd(reinterpret_cast<unsigned long long*>(&totals[0]), (unsigned long long)a0);
+        if (a1) atomicAdd(reinterpret_cast<unsigned long long*>(&totals[1]), (unsigned long long)a1);
+    }
+}
+
+// ---- per-token scatter ------------------------------------------------------
+
+__global__ void scatter_kernel(SegArgs a) {
+    const int64_t nv = a.totals_in[0];
+    const int64_t rv = a.totals_in[1];
+    const int32_t S = a.num_segs;
+    for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < a.N; k += (int64_t)gridDim.x * blockDim.x) {
+        float adv = 0.f, w = 0.f;
+        if (S > 0 && k >= a.seg_offsets[0] && k < a.seg_offsets[S]) {
+            // Last s with seg_offsets[s] <= k (upper bound - 1).
+            int32_t lo = 0, hi = S;  // search in [lo, hi)
+            while (hi - lo > 1) {
+                const int32_t mid = (lo + hi) >> 1;
+                if (a.seg_offsets[mid] <= k) lo = mid; else hi = mid;
+            }
+            int32_t a0, b0, i, t;
+            if (segment_ok(a, lo, a0, b0, i, t) && k >= a0 && k < b0 && t >= 0 && t < (int)a.T_eff[i]) {
+                adv = a.turn_adv[(int64_t)i * a.M + t];
+                if (a.agg == 1) {
+                    w = nv > 0 ? (float)(1.0 / (double)nv) : 0.f;
+                } else {
+                    const int32_t L = a.L_in[i];
+                    w = (rv > 0 && L > 0) ? (float)(1.0 / ((double)rv * (double)L)) : 0.f;
+                }
+            }
+        }
+        a.adv_out[k] = adv;
+        a.w_out[k] = w;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_rank_advantages(const RankArgs& a, cudaStream_t s) {
+    if (a.num_groups == 0) return cudaSuccess;
+    const int J = (a.G + 31) / 32;
+    if (J <= 1) return launch_rank_j<1>(a, s);
+    if (J <= 2) return launch_rank_j<2>(a, s);
+    if (J <= 4) return launch_rank_j<4>(a, s);
+    if (J <= 8) return launch_rank_j<8>(a, s);
+    if (J <= 16) return launch_rank_j<16>(a, s);
+    return launch_rank_j<32>(a, s);
+}
+
+cudaError_t launch_token_counts(const SegArgs& a, cudaStream_t s) {
+    const int sms = device_sm_count();
+    const int64_t zb = std::min<int64_t>(((int64_t)a.n_rollouts + 255) / 256, (int64_t)sms * 4);
+    zero_counts_kernel<<<(unsigned)std::max<int64_t>(zb, 1), 256, 0, s>>>(a.L_out, a.n_rollouts, a.totals_out);
+    if (a.num_segs > 0) {
+        segment_count_kernel<<<(unsigned)(((int64_t)a.num_segs + 255) / 256), 256, 0, s>>>(a);
+    }
+    if (a.n_rollouts > 0) {
+        totals_kernel<<<(unsigned)std::max<int64_t>(zb, 1), 256, 0, s>>>(a.L_out, a.n_rollouts, a.totals_out);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_scatter(const SegArgs& a, cudaStream_t s) {
+    if (a.N == 0) return cudaSuccess;
+    const int sms = device_sm_count();
+    const int64_t blocks = std::min<int64_t>((a.N + 255) / 256, (int64_t)sms * 8);
+    scatter_kernel<<<(unsigned)blocks, 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace leap

@@ -1,0 +1,84 @@
+"""One pass of the LEAP loss hot path over a resident batch, through libleap.
+
+GrpoStep owns the device buffers of one batch shape and runs, on the current
+stream:
+  1. leap_group_rank_advantages    DCP gate, tiers, tournament, R, A, A_hat (Sec. 3.1-3.3)
+  2. leap_rollout_token_counts     per-rollout optimised-token counts, local totals
+  3. (data parallel) all_reduce(totals)  the one exchange: global loss normalisers
+  4. leap_scatter_turn_advantages  per-token advantage and aggregation weight
+  5. leap_grpo_loss_fwd            clipped surrogate + fused dlogits (Eq. 3)
+Only step 3 leaves libleap, and only when a process group with more than one
+rank is passed in.
+"""
+
+from __future__ import annotations
+
+import torch
+
+from . import leap as L
+
+
+class GrpoStep:
+    def __init__(self, batch, V, device, *, gamma=0.9, tau=None, use_gate_in=True, eps_std=1e-6,
+                 eps_low=0.2, eps_high=0.2, inv_temp=1.0, grad_scale=1.0, agg=L.LEAP_AGG_SEQ_MEAN_TOKEN_MEAN,
+                 chunk_rows=None):
+        self.b = batch
+        self.V = int(V)
+        self.dev = torch.device(device)
+        self.gamma, self.eps_std = gamma, eps_std
+        self.tau = tau if tau is not None else (0, batch.G)
+        self.use_gate_in = use_gate_in and batch.gate_in is not None
+        self.loss_kw = dict(eps_low=eps_low, eps_high=eps_high, inv_temp=inv_temp, grad_scale=grad_scale)
+        self.agg = agg
+        n, N, M = batch.n, batch.N, batch.M
+        d = self.dev
+        as_dev = lambda x, dt: torch.as_tensor(x).to(dt).to(d)
+        # Per-batch structure (inputs).
+        self.pass_turn = as_dev(batch.pass_turn, torch.int8)
+        self.num_turns = as_dev(batch.num_turns, torch.int8)
+        self.gate_in = as_dev(batch.gate_in, torch.uint8) if self.use_gate_in else None
+        self.seg_offsets = as_dev(batch.seg_offsets, torch.int32)
+        self.seg_rollout = as_dev(batch.seg_rollout, torch.int32)
+        self.seg_turn = as_dev(batch.seg_turn, torch.int8)
+        # Intermediates and outputs.
+        e = lambda shape, dt: torch.empty(shape, dtype=dt, device=d)
+        self.rank_out = dict(gate=e(batch.num_groups, torch.uint8), r=e(n, torch.uint8),
+                             n_worse=e(n, torch.int32), n_better=e(n, torch.int32), R=e(n, torch.float32),
+                             A=e(n, torch.float32), turn_adv=e(n * M, torch.float32), T_eff=e(n, torch.uint8))
+        self.L = e(n, torch.int32)
+        self.totals = e(2, torch.int64)
+        self.adv = e(N, torch.float32)
+        self.w = e(N, torch.float32)
+        self.loss = e(1, torch.float32)
+        self.chunk_rows = int(chunk_rows) if chunk_rows else N
+        self.workspace = L.loss_workspace(min(N, self.chunk_rows), self.V, d)
+
+    def advantages(self, pg=None):
+        """Steps 1-4: per-token advantages and weights."""
+        b = self.b
+        L.leap_group_rank_advantages(self.pass_turn, self.num_turns, G=b.G, M=b.M, tau_min=self.tau[0],
+                                     tau_max=self.tau[1], gamma=self.gamma, eps_std=self.eps_std,
+                                     gate_in=self.gate_in, out=self.rank_out)
+        L.leap_rollout_token_counts(b.N, self.seg_offsets, self.seg_rollout, self.seg_turn,
+                                    self.rank_out["T_eff"], M=b.M, L=self.L, totals=self.totals)
+        if pg is not None and torch.distributed.get_world_size(pg) > 1:
+            torch.distributed.all_reduce(self.totals, group=pg)
+        L.leap_scatter_turn_advantages(b.N, self.seg_offsets, self.seg_rollout, self.seg_turn,
+                                       self.rank_out["turn_adv"], self.rank_out["T_eff"], self.L, self.totals,
+                                       M=b.M, agg=self.agg, adv=self.adv, w=self.w)
+
+    def loss_pass(self, logits, ids, old_logp, dlogits, row0=0, accumulate=False, stats=None):
+        """Step 5 over rows [row0, row0 + logits.shape[0]) of the packed stream."""
+        n = logits.shape[0]
+        return L.leap_grpo_loss_fwd(logits, ids, old_logp, self.adv[row0:row0 + n], self.w[row0:row0 + n],
+                                    V=self.V, loss=self.loss, dlogits=dlogits, want_outputs=False,
+                                    workspace=self.workspace, accumulate=accumulate, stats=stats, **self.loss_kw)
+
+    def run(self, logits, ids, old_logp, dlogits, pg=None):
+        """The whole pass for a batch whose logits are all resident."""
+        self.advantages(pg)
+        self.loss_pass(logits, ids, old_logp, dlogits)
+        return self.loss
+
+    # Kernel launches one run() makes (rank 1, counts 3, scatter 1, loss 1 + reduce 2).
+    LAUNCHES_PER_RUN = 8

@@ -1,0 +1,129 @@
+"""End-to-end parity of the whole hot path (rank advantages -> token counts ->
+scatter -> fused loss fwd+bwd) on the benchmark workloads, each side running
+its own pipeline from the same raw outcomes, layout and logits."""
+import numpy as np
+import pytest
+import torch
+
+from harness import (O, TOL_ADV, TOL_LOGP, TOL_LOSS_REL, bf16_rows_to_f64, check_dlogits_rows, leap,
+                     oracle_rank, oracle_tokens, rows_f64, to_dev, torch_logp)
+from paper_2608_01804_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+def _gpu_pipeline(L, b, z, ids, old, V, gamma, tau, use_gate_in, agg=0, grad_scale=1.0):
+    dev = "cuda"
+    pt, nt = to_dev(b.pass_turn, torch.int8), to_dev(b.num_turns, torch.int8)
+    gi = to_dev(b.gate_in, torch.uint8) if (use_gate_in and b.gate_in is not None) else None
+    rk = L.leap_group_rank_advantages(pt, nt, G=b.G, M=b.M, tau_min=tau[0], tau_max=tau[1], gamma=gamma,
+                                      gate_in=gi)
+    so, sr, st = to_dev(b.seg_offsets, torch.int32), to_dev(b.seg_rollout, torch.int32), to_dev(b.seg_turn, torch.int8)
+    Lc, tot = L.leap_rollout_token_counts(b.N, so, sr, st, rk["T_eff"], M=b.M)
+    adv, w = L.leap_scatter_turn_advantages(b.N, so, sr, st, rk["turn_adv"], rk["T_eff"], Lc, tot, M=b.M, agg=agg)
+    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, grad_scale=grad_scale)
+    return rk, adv, w, out
+
+
+def _oracle_pipeline(b, gamma, tau, use_gate_in, agg=0):
+    orc = oracle_rank(b, tau=tau, gamma=gamma, use_gate_in=use_gate_in)
+    ta = orc["turn_adv"].reshape(-1)
+    T_eff = orc["T_eff"].reshape(-1)
+    _, _, _, adv, w = oracle_tokens(b, ta, T_eff, agg)
+    return orc, adv, w
+
+
+@pytest.mark.parametrize("use_gate_in,tau", [(True, (0, 8)), (False, (4, 7))])
+def test_tiny_workload_all_rows(use_gate_in, tau):
+    """4 prompts x 8 x 2 turns x 256, V = 1024: every row and every output."""
+    L = leap()
+    b = synth.tiny_batch()
+    V = 1024
+    z = synth.logits(b.N, V, 2.0, 100, "cuda")
+    ids = synth.token_ids(b.N, V, 101, "cuda")
+    old = torch_logp(z, ids, V) + synth.normal(b.N, 0.05, 102, "cuda")
+    rk, adv, w, out = _gpu_pipeline(L, b, z, ids, old, V, 0.9, tau, use_gate_in, grad_scale=1000.0)
+    orc, adv_o, w_o = _oracle_pipeline(b, 0.9, tau, use_gate_in)
+    np.testing.assert_array_equal(rk["n_worse"].cpu().numpy(), orc["n_worse"].reshape(-1))
+    assert np.max(np.abs(adv.cpu().numpy() - adv_o)) <= TOL_ADV
+    np.testing.assert_allclose(w.cpu().numpy(), w_o, rtol=2e-7)
+    res = O.grpo_loss_rows(rows_f64(z, range(b.N), V), ids.cpu().numpy(), old.cpu().numpy().astype(np.float64),
+                           adv_o, w_o, grad_scale=1000.0)
+    assert np.max(np.abs(out["logp"].cpu().numpy() - res["logp"])) <= TOL_LOGP
+    assert abs(out["loss"].item() - res["loss"]) <= TOL_LOSS_REL * abs(res["loss"])
+    check_dlogits_rows(bf16_rows_to_f64(out["dlogits"]), res, list(range(b.N)))
+
+
+def test_single_turn_workload_full_size_sampled():
+    """16 x 8 x 256 = 32,768 rows at V = 151,936 in the benchmark's launch
+    configuration; sampled rows against the oracle, the loss against the fp64
+    sum of the kernel's own per-row terms and against the oracle's terms on the
+    sampled rows."""
+    L = leap()
+    b = synth.single_turn_batch()
+    V = 151936
+    z = synth.logits(b.N, V, 3.0, 200, "cuda", spike_frac=0.01)
+    ids = synth.token_ids(b.N, V, 201, "cuda")
+    old = torch_logp(z, ids, V) + synth.normal(b.N, 0.05, 202, "cuda")
+    rk, adv, w, out = _gpu_pipeline(L, b, z, ids, old, V, 1.0, (0, b.G), False)
+    orc, adv_o, w_o = _oracle_pipeline(b, 1.0, (0, b.G), False)
+    assert np.max(np.abs(adv.cpu().numpy() - adv_o)) <= TOL_ADV
+    rng = np.random.default_rng(0)
+    rows = sorted(set([0, 1, b.N - 1, b.N - 2] + list(rng.choice(b.N, 96, replace=False))))
+    sel = torch.as_tensor(rows, device="cuda")
+    res = O.grpo_loss_rows(rows_f64(z, rows, V), ids[sel].cpu().numpy(), old[sel].cpu().numpy().astype(np.float64),
+                           adv_o[rows], w_o[rows])
+    logp = out["logp"][sel].cpu().numpy()
+    assert np.max(np.abs(logp - res["logp"])) <= TOL_LOGP
+    ell = out["ell"][sel].cpu().numpy().astype(np.float64)
+    np.testing.assert_allclose(ell, res["ell"], rtol=1e-4, atol=1e-6)
+    check_dlogits_rows(bf16_rows_to_f64(out["dlogits"][sel]), res, rows)
+    # Reduction: the loss is the fp64 sum of w * ell over all rows.
+    tot = float((w.double() * out["ell"].double()).sum().item())
+    assert abs(out["loss"].item() - tot) <= 1e-6 * abs(tot) + 1e-12
+    # Masked padding rows: zero dlogits.
+    masked = (w == 0).nonzero().view(-1)[:64]
+    assert torch.all(out["dlogits"][masked] == 0)
+
+
+def test_multiturn_dcp_workload_chunked():
+    """The packed multi-turn batch (~1M tokens) streamed through one 65,536-row
+    logits chunk buffer with loss accumulation; three chunks are checked against
+    the oracle on sampled rows, the advantages and weights on every token."""
+    L = leap()
+    b = synth.multiturn_dcp_batch()
+    V, CH = 151936, 65536
+    pt, nt = to_dev(b.pass_turn, torch.int8), to_dev(b.num_turns, torch.int8)
+    rk = L.leap_group_rank_advantages(pt, nt, G=b.G, M=b.M, tau_min=8, tau_max=15, gamma=0.9)
+    np.testing.assert_array_equal(rk["gate"].cpu().numpy(), b.gate_in)   # the drawn zone matches Eq. 2
+    so, sr, st = to_dev(b.seg_offsets, torch.int32), to_dev(b.seg_rollout, torch.int32), to_dev(b.seg_turn, torch.int8)
+    Lc, tot = L.leap_rollout_token_counts(b.N, so, sr, st, rk["T_eff"], M=b.M)
+    adv, w = L.leap_scatter_turn_advantages(b.N, so, sr, st, rk["turn_adv"], rk["T_eff"], Lc, tot, M=b.M)
+    orc, adv_o, w_o = _oracle_pipeline(b, 0.9, (8, 15), False)
+    assert np.max(np.abs(adv.cpu().numpy() - adv_o)) <= TOL_ADV
+    np.testing.assert_allclose(w.cpu().numpy(), w_o, rtol=2e-7)
+    z = synth.logits(CH, V, 3.0, 300, "cuda", spike_frac=0.01)
+    ids_all = synth.token_ids(b.N, V, 301, "cuda")
+    loss = torch.zeros(1, device="cuda")
+    dl = torch.empty_like(z)
+    ws = L.loss_workspace(CH, V, "cuda")
+    nchunks = -(-b.N // CH)
+    total_o = 0.0
+    for c in range(nchunks):
+        a0, a1 = c * CH, min(b.N, (c + 1) * CH)
+        n = a1 - a0
+        ids = ids_all[a0:a1].contiguous()
+        old = torch_logp(z[:n], ids, V) + synth.normal(n, 0.05, 400 + c, "cuda")
+        out = L.leap_grpo_loss_fwd(z[:n], ids, old, adv[a0:a1].contiguous(), w[a0:a1].contiguous(), V=V, loss=loss,
+                                   accumulate=True, dlogits=dl[:n], workspace=ws)
+        if c in (0, nchunks // 2, nchunks - 1):
+            rng = np.random.default_rng(c)
+            live = np.nonzero(w_o[a0:a1])[0]
+            rows = sorted(set(rng.choice(live, min(24, len(live)), replace=False).tolist() + [0, n - 1]))
+            sel = torch.as_tensor(rows, device="cuda")
+            res = O.grpo_loss_rows(rows_f64(z, rows, V), ids[sel].cpu().numpy(),
+                                   old[sel].cpu().numpy().astype(np.float64), adv_o[a0:a1][rows], w_o[a0:a1][rows])
+            assert np.max(np.abs(out["logp"][sel].cpu().numpy() - res["logp"])) <= TOL_LOGP
+            check_dlogits_rows(bf16_rows_to_f64(dl[sel]), res, rows)
+        total_o += float((out["ell"].double() * w[a0:a1].double()).sum().item())
+    assert abs(loss.item() - total_o) <= 1e-5 * abs(total_o) + 1e-9

@@ -1,0 +1,115 @@
+"""GPU parity: rank-based advantages (Sec. 3.1-3.3) against the oracle.
+
+Integers, the gate and R are compared bit for bit; A and the per-turn
+advantages within 1e-5 absolute."""
+import numpy as np
+import pytest
+import torch
+
+from harness import O, TOL_ADV, leap, oracle_rank, to_dev
+from paper_2608_01804_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+def _run_gpu(pass_turn, num_turns, G, M, tau, gamma, gate_in=None, **kw):
+    L = leap()
+    return L.leap_group_rank_advantages(to_dev(pass_turn, torch.int8), to_dev(num_turns, torch.int8), G=G, M=M,
+                                        tau_min=tau[0], tau_max=tau[1], gamma=gamma,
+                                        gate_in=None if gate_in is None else to_dev(gate_in, torch.uint8), **kw)
+
+
+def _compare(gpu, orc, M, strict_A=True):
+    n = orc["r"].size
+    np.testing.assert_array_equal(gpu["gate"].cpu().numpy(), orc["gate"])
+    np.testing.assert_array_equal(gpu["r"].cpu().numpy(), orc["r"].reshape(-1))
+    np.testing.assert_array_equal(gpu["T_eff"].cpu().numpy(), orc["T_eff"].reshape(-1))
+    np.testing.assert_array_equal(gpu["n_worse"].cpu().numpy(), orc["n_worse"].reshape(-1))
+    np.testing.assert_array_equal(gpu["n_better"].cpu().numpy(), orc["n_better"].reshape(-1))
+    R32 = orc["R"].reshape(-1).astype(np.float32)
+    np.testing.assert_array_equal(gpu["R"].cpu().numpy(), R32)
+    A = gpu["A"].cpu().numpy().astype(np.float64)
+    assert np.max(np.abs(A - orc["A"].reshape(-1))) <= TOL_ADV
+    ta = gpu["turn_adv"].cpu().numpy().astype(np.float64).reshape(n, M)
+    assert np.max(np.abs(ta - orc["turn_adv"].reshape(n, M))) <= TOL_ADV
+    # Signs decide the discount base: they must agree exactly where A != 0.
+    nz = orc["A"].reshape(-1) != 0
+    assert np.all(np.sign(A[nz]) == np.sign(orc["A"].reshape(-1)[nz]))
+
+
+def test_tiny_batch_recorded_gate():
+    b = synth.tiny_batch()
+    gpu = _run_gpu(b.pass_turn, b.num_turns, b.G, b.M, (0, b.G), 0.9, gate_in=b.gate_in)
+    orc = oracle_rank(b, gamma=0.9)
+    _compare(gpu, orc, b.M)
+    # Turn 2 of the gated-off prompts 0 and 1 is pruned.
+    assert np.all(gpu["T_eff"].cpu().numpy()[:16] == 1)
+
+
+@pytest.mark.parametrize("tau", [(4, 7), (0, 8), (8, 8), (0, 0)])
+def test_tiny_batch_computed_gate(tau):
+    b = synth.tiny_batch(seed=5)
+    gpu = _run_gpu(b.pass_turn, b.num_turns, b.G, b.M, tau, 0.5)
+    orc = oracle_rank(b, tau=tau, gamma=0.5, use_gate_in=False)
+    _compare(gpu, orc, b.M)
+
+
+def test_tournament_stress_full_size():
+    """65,536 groups x G = 64, M = 3, ~10% exact duplicate tuples: bit-exact counts."""
+    pt, nt, sp, tok = synth.tournament_outcomes()
+    G, M = 64, 3
+    gpu = _run_gpu(pt, nt, G, M, (50, 56), 0.9)
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, 50, 56, 0.9)
+    _compare(gpu, orc, M)
+    assert 0.2 < orc["gate"].mean() < 0.9
+
+
+@pytest.mark.parametrize("G", [2, 3, 31, 32, 33, 64, 100, 257, 1024])
+@pytest.mark.parametrize("M", [1, 3, 8])
+def test_group_sizes_and_turns(G, M):
+    rng = np.random.default_rng(G * 10 + M)
+    groups = max(1, 4096 // G)
+    nt = rng.integers(1, M + 1, size=groups * G).astype(np.int8)
+    pt = np.where(rng.random(groups * G) < 0.5, rng.integers(1, M + 1, size=groups * G), 0)
+    pt = np.minimum(pt, nt).astype(np.int8)
+    tau = (G // 4, (3 * G) // 4)
+    gpu = _run_gpu(pt, nt, G, M, tau, 0.8)
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, tau[0], tau[1], 0.8)
+    _compare(gpu, orc, M)
+
+
+@pytest.mark.parametrize("norm,unbiased,eps", [(O.ADVNORM_NONE, 1, 1e-6), (O.ADVNORM_GRPO_STD, 0, 1e-6),
+                                                (O.ADVNORM_GRPO_STD, 1, 0.0), (O.ADVNORM_GRPO_STD, 1, 0.1)])
+def test_norm_modes(norm, unbiased, eps):
+    b = synth.multiturn_dcp_batch(seed=7)
+    gpu = _run_gpu(b.pass_turn, b.num_turns, b.G, b.M, (0, b.G), 0.9, gate_in=b.gate_in, norm=norm,
+                   std_unbiased=bool(unbiased), eps_std=eps)
+    orc = oracle_rank(b, gamma=0.9, eps_std=eps, norm=norm, std_unbiased=bool(unbiased))
+    _compare(gpu, orc, b.M)
+
+
+def test_bad_outcomes_flagged_and_ranked_as_failures():
+    L = leap()
+    L.leap_get_device_status()
+    G, M = 8, 2
+    pt = np.array([1, 2, 0, 5, 1, 1, -1, 2], dtype=np.int8)
+    nt = np.array([1, 2, 2, 2, 1, 1, 1, 1], dtype=np.int8)   # index 7: pass at 2 > T = 1
+    gpu = _run_gpu(pt, nt, G, M, (0, G), 0.9)
+    orc = O.rank_advantages(pt.reshape(1, G), nt.reshape(1, G), M, 0, G, 0.9)
+    _compare(gpu, orc, M)
+    assert L.leap_get_device_status() & L.LEAP_DEV_BAD_OUTCOME
+    assert L.leap_get_device_status() == 0   # cleared by the read
+
+
+def test_empty_and_gamma_one():
+    L = leap()
+    empty = torch.empty(0, dtype=torch.int8, device="cuda")
+    out = L.leap_group_rank_advantages(empty, empty, G=8, M=2, tau_max=8)
+    assert out["A"].numel() == 0
+    b = synth.tiny_batch(seed=9)
+    gpu = _run_gpu(b.pass_turn, b.num_turns, b.G, b.M, (0, b.G), 1.0, gate_in=b.gate_in)
+    ta = gpu["turn_adv"].cpu().numpy().reshape(-1, b.M)
+    T = gpu["T_eff"].cpu().numpy()
+    A = gpu["A"].cpu().numpy()
+    for i in range(ta.shape[0]):
+        assert np.all(ta[i, :T[i]] == A[i]) and np.all(ta[i, T[i]:] == 0)
