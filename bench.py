@@ -57,6 +57,8 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--prompts", type=int, default=16,
+                    help="prompts per rank (16 = the benchmark workload; fewer only for profiling captures)")
     return ap.parse_args()
 
 
@@ -139,9 +141,9 @@ def torch_logp(logits, ids, chunk=2048):
     return out
 
 
-def make_inputs(rank, device):
+def make_inputs(rank, device, prompts=16):
     from paper_2608_01804_gb300 import synth
-    batch = synth.single_turn_batch(seed=1 + 1000 * rank)
+    batch = synth.single_turn_batch(seed=1 + 1000 * rank, num_prompts=prompts)
     N = batch.N
     logits = synth.logits(N, V, 3.0, 200 + rank, device, spike_frac=0.01)
     ids = synth.token_ids(N, V, 201 + rank, device)
@@ -244,7 +246,7 @@ def main():
     build.build()
     from paper_2608_01804_gb300.step import GrpoStep
 
-    batch, logits, ids, old = make_inputs(rank, device)
+    batch, logits, ids, old = make_inputs(rank, device, args.prompts)
     N = batch.N
     n_valid = valid_tokens(batch)
     step = GrpoStep(batch, V, device, gamma=1.0, tau=(0, batch.G), use_gate_in=False)
@@ -346,7 +348,8 @@ def main():
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
                 "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "f32", "data": "synthetic",
-                "config": {"workload": WORKLOAD, "rows_per_step_per_gpu": N, "valid_tokens_per_step_per_gpu": n_valid,
+                "config": {"workload": WORKLOAD if args.prompts == 16 else "%d-prompt slice of: %s" % (args.prompts, WORKLOAD),
+                           "rows_per_step_per_gpu": N, "valid_tokens_per_step_per_gpu": n_valid,
                            "vocab": V, "logits_dtype": "bf16", "l2": "inputs larger than L2 (9.96 GB of logits "
                            "read and 9.96 GB of dlogits written per step)", "parallelism": "dp%d" % world},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,

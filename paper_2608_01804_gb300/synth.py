@@ -81,6 +81,7 @@ def padded_batch(num_prompts, G, M, slot_len, pass_prob, len_lo, len_hi, seed, g
             num_turns[i] = hit[0] + 1
     segs = []
     ntok = np.zeros(n, dtype=np.int32)
+    starts = np.arange(n + 1, dtype=np.int64) * (M * slot_len)
     for i in range(n):
         for t in range(M):
             if t < num_turns[i]:
@@ -93,7 +94,7 @@ def padded_batch(num_prompts, G, M, slot_len, pass_prob, len_lo, len_hi, seed, g
     so, sr, st = _segments_to_arrays(segs)
     gi = None if gate_in is None else np.asarray(gate_in, dtype=np.uint8)
     return RolloutBatch(num_prompts, G, M, pass_turn, num_turns, speed, ntok, gi, int(so[-1]), so, sr, st,
-                        info=dict(layout="padded", slot_len=slot_len))
+                        info=dict(layout="padded", slot_len=slot_len, rollout_starts=starts))
 
 
 def tiny_batch(seed=0):
@@ -101,9 +102,9 @@ def tiny_batch(seed=0):
     return padded_batch(4, 8, 2, 256, 0.4, 64, 256, seed, gate_in=[0, 0, 1, 1])
 
 
-def single_turn_batch(seed=1):
+def single_turn_batch(seed=1, num_prompts=16):
     """16 prompts x G=8 x 256 tokens (32,768 rows), one turn, pass ~ Bernoulli(0.3)."""
-    return padded_batch(16, 8, 1, 256, 0.3, 64, 256, seed, gate_in=None)
+    return padded_batch(num_prompts, 8, 1, 256, 0.3, 64, 256, seed, gate_in=None)
 
 
 def multiturn_dcp_batch(seed=2, num_prompts=32, G=16, M=3, len_lo=256, len_hi=2048, frac_expanded=0.4,
@@ -148,16 +149,44 @@ def multiturn_dcp_batch(seed=2, num_prompts=32, G=16, M=3, len_lo=256, len_hi=20
     speed = rng.lognormal(0.0, 0.5, size=n).astype(np.float32)
     segs = []
     ntok = np.zeros(n, dtype=np.int32)
+    starts = np.zeros(n + 1, dtype=np.int64)
+    cur = 0
     for i in range(n):
+        starts[i] = cur
         for t in range(int(num_turns[i])):
             if t > 0:
-                segs.append((int(rng.integers(len_lo, len_hi + 1)), -1, -1))
+                fb = int(rng.integers(len_lo, len_hi + 1))
+                segs.append((fb, -1, -1))
+                cur += fb
             ln = int(rng.integers(len_lo, len_hi + 1))
             segs.append((ln, i, t))
             ntok[i] += ln
+            cur += ln
+    starts[n] = cur
     so, sr, st = _segments_to_arrays(segs)
     return RolloutBatch(num_prompts, G, M, pass_turn, num_turns, speed, ntok, expanded, int(so[-1]), so, sr, st,
-                        info=dict(layout="packed", expanded_prompts=int(n_exp), tau=tau))
+                        info=dict(layout="packed", expanded_prompts=int(n_exp), tau=tau, rollout_starts=starts))
+
+
+def shard(batch, rank, world):
+    """The rollout groups [g0, g1) of this rank (contiguous split) with their
+    tokens: segment offsets re-based to the shard, rollout indices local."""
+    per = -(-batch.num_groups // world)
+    g0, g1 = min(batch.num_groups, rank * per), min(batch.num_groups, (rank + 1) * per)
+    i0, i1 = g0 * batch.G, g1 * batch.G
+    starts = batch.info["rollout_starts"]
+    t0, t1 = int(starts[i0]), int(starts[i1])
+    so = batch.seg_offsets
+    s0 = int(np.searchsorted(so, t0, side="left"))
+    s1 = int(np.searchsorted(so, t1, side="left"))
+    seg_offsets = (so[s0:s1 + 1] - t0).astype(np.int32)
+    sr = batch.seg_rollout[s0:s1].copy()
+    sr[sr >= 0] -= i0
+    info = dict(batch.info, rollout_starts=starts[i0:i1 + 1] - t0, shard=(g0, g1), token_range=(t0, t1))
+    return RolloutBatch(g1 - g0, batch.G, batch.M, batch.pass_turn[i0:i1], batch.num_turns[i0:i1],
+                        batch.speedup[i0:i1], batch.ntokens[i0:i1],
+                        None if batch.gate_in is None else batch.gate_in[g0:g1], t1 - t0, seg_offsets, sr,
+                        batch.seg_turn[s0:s1].copy(), info=info)
 
 
 def tournament_outcomes(seed=3, num_groups=65536, G=64, M=3, dup_frac=0.1):

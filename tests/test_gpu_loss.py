@@ -19,7 +19,7 @@ def _inputs(N, V, seed, sigma=2.0, spikes=0.0, old_sigma=0.05, ld=None, mask_fra
     old = torch_logp(z, ids, V) + synth.normal(N, old_sigma, seed + 2, dev)
     rng = np.random.default_rng(seed + 3)
     adv = torch.as_tensor(rng.normal(0, adv_scale, N).astype(np.float32), device=dev)
-    w = rng.uniform(0.5, 2.0, N).astype(np.float32)
+    w = rng.uniform(0.01, 0.1, N).astype(np.float32)
     w[rng.random(N) < mask_frac] = 0.0
     return z, ids, old, adv, torch.as_tensor(w, device=dev)
 
@@ -52,7 +52,7 @@ def test_fused_loss_all_rows(V, ld):
     N = 64 if V > 50000 else 256
     z, ids, old, adv, w = _inputs(N, V, seed=V % 97, sigma=3.0, spikes=0.01, ld=ld, old_sigma=0.3)
     ids[:4] = torch.tensor([0, V - 1, min(7, V - 1), min(8, V - 1)], dtype=torch.int32, device="cuda")
-    w[:4] = 1.0
+    w[:4] = 0.1
     if ld > V:
         sentinel = torch.full((N, ld - V), 3.0, dtype=torch.bfloat16, device="cuda")
     out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, dlogits=torch.full_like(z, 3.0) if ld > V else None)
