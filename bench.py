@@ -257,9 +257,14 @@ def main():
         if pg is not None:
             torch.distributed.barrier()
 
+    from paper_2608_01804_gb300 import leap as L
+    L.leap_get_device_status()
     for _ in range(max(3, args.warmup)):
         step.run(logits, ids, old, dlogits, pg)
     torch.cuda.synchronize()
+    flags = L.leap_get_device_status()
+    if flags:
+        raise RuntimeError("libleap device status 0x%x after the warm-up steps" % flags)
     live_rows = int((step.w != 0).sum().item())
     assert live_rows == n_valid
 

@@ -27,8 +27,10 @@
  *  - bf16 tensors are passed as uint16_t bit patterns.  Row-major matrices
  *    have a leading dimension `ld` (elements); bf16 matrices need a 16-byte
  *    aligned base and ld % 8 == 0.
- *  - No kernel spins on a flag or waits on another launch; nothing here can
- *    time out.
+ *  - No kernel waits on another launch.  The fused loss kernel waits on its
+ *    own asynchronous copies and on the other CTAs of its cluster through
+ *    mbarriers; every such wait is bounded and, if it ever gave up, the
+ *    kernel would set LEAP_DEV_TIMEOUT and finish instead of hanging.
  */
 #ifndef LEAP_H_
 #define LEAP_H_
@@ -45,7 +47,7 @@ typedef enum {
     LEAP_ERR_INVALID_ARG = 1,
     LEAP_ERR_UNSUPPORTED = 2,
     LEAP_ERR_CUDA = 3,
-    LEAP_ERR_TIMEOUT = 4,     /* reserved: no current kernel can time out */
+    LEAP_ERR_TIMEOUT = 4,     /* reserved (a wait that gave up is reported as LEAP_DEV_TIMEOUT) */
     LEAP_ERR_BAD_INDEX = 5    /* returned by leap_get_device_status() when a bit is set */
 } leap_status_t;
 
@@ -53,6 +55,7 @@ typedef enum {
 #define LEAP_DEV_BAD_ID 1u      /* a token id with nonzero weight lay outside [0, V) */
 #define LEAP_DEV_BAD_OUTCOME 2u /* pass_turn / num_turns out of range or inconsistent */
 #define LEAP_DEV_BAD_SEGMENT 4u /* segment offsets, rollout or turn out of range */
+#define LEAP_DEV_TIMEOUT 8u     /* a bounded wait inside a kernel gave up (results undefined) */
 
 /* Human-readable name of a status code (static storage). */
 const char* leap_status_string(leap_status_t status);
@@ -229,7 +232,7 @@ size_t leap_grpo_loss_workspace_size(int64_t N, int32_t V);
  * dlogits bf16 [N x ld] (optional; columns >= V untouched); stats optional.
  * workspace: >= leap_grpo_loss_workspace_size(N, V) bytes, 256-byte aligned,
  * contents ignored on entry.  Requires 1 <= V; the fused backward supports
- * V up to 1,048,576 (LEAP_ERR_UNSUPPORTED beyond: use the split path).
+ * V up to 262,144 (LEAP_ERR_UNSUPPORTED beyond: use the split path).
  */
 leap_status_t leap_grpo_loss_fwd(
     const leap_loss_params_t* params,

@@ -214,112 +214,210 @@ __global__ void __launch_bounds__(512) row_stream_kernel(RowArgs a, int mode) {
 }
 
 // ---------------------------------------------------------------------------
-// Fused forward + backward.  Grid = N * C CTAs; the C consecutive CTAs of a
-// cluster share one row.  CTA c owns 16-byte vectors [c * per, (c+1) * per)
-// of the row (per = ceil(V8 / C) <= T * NV) and holds them in registers
-// between the forward reduction and the dlogits write.
+// Fused forward + backward, persistent.  A cluster of C CTAs owns one row at a
+// time and walks rows cid, cid + ncl, cid + 2 ncl, ...; CTA c owns 16-byte
+// vectors [c * per, (c+1) * per) of every row.  Per CTA:
+//   * a producer warp reads the weights / ids of the next 32 rows of the
+//     sequence at once and, for each live row, issues a 1-D bulk async copy
+//     (TMA) of the CTA's slice plus the 16-byte vector holding the target logit
+//     into one of STAGES shared-memory stages (mbarrier full/empty pipeline);
+//   * T consumer threads copy a ready stage into registers (NV vectors each),
+//     release it at once, reduce it to (max, sum of 2^((z - max) log2e)), push
+//     that pair to every CTA of the cluster through distributed shared memory
+//     with a remote mbarrier arrive, merge the C pairs, and write the dlogits
+//     slice straight from the registers they still hold.
+// Logits are read from HBM once and dlogits written once.  Masked rows skip
+// the copy and write zeros.  Every wait is bounded (LEAP_DEV_TIMEOUT).
 // ---------------------------------------------------------------------------
-template <int C, int T, int NV>
-__global__ void __launch_bounds__(T) fused_loss_kernel(RowArgs a) {
-    __shared__ float2 wpart[T / 32];
-    __shared__ float2 cta_part;  // read by the other CTAs of the cluster
-    __shared__ float bc[2];
+template <int STAGES, int C>
+struct FusedSmem {
+    uint64_t full[STAGES];
+    uint64_t empty[STAGES];
+    uint64_t ex[2];          // exchange barriers (C arrivals each), alternating per live row
+    float2 slot[2][C];       // (max, sum) of each CTA of the cluster, alternating per live row
+    float2 wpart[32];
+    float bc[2];
+    uint4 yvec[STAGES];      // the 16-byte vector that holds the target logit
+    int abort_flag;          // set once a bounded wait of this CTA gave up
+};
+
+template <int C, int T, int NV, int STAGES>
+__global__ void __launch_bounds__(T + 32) fused_loss_kernel(RowArgs a, int32_t per, int32_t ncl) {
+    extern __shared__ __align__(128) uint4 stage_mem[];  // STAGES * per vectors
+    __shared__ __align__(16) FusedSmem<STAGES, C> sm;
+    const int t = threadIdx.x;
     const uint32_t crank = (C > 1) ? cluster_ctarank() : 0u;
-    const int64_t row = blockIdx.x / C;
-    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int64_t cid = blockIdx.x / C;
     const int V = a.V;
     const int64_t V8 = ((int64_t)V + 7) >> 3;
-    const int64_t per = (V8 + C - 1) / C;
-    const int64_t vbeg = (int64_t)crank * per;
+    const int64_t vbeg = min((int64_t)crank * per, V8);
     const int64_t vend = min(vbeg + per, V8);
+    const uint32_t nvec = (uint32_t)(vend - vbeg);
     const int tailn = V & 7;
-    const float wk = a.w[row];
-    const int id = a.ids[row];
-    const bool bad = (wk != 0.f) && (id < 0 || id >= V);
-    uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
 
-    if (wk == 0.f || bad) {  // masked row: the same branch for the whole cluster
+    if (t == 0) {
 #pragma unroll
-        for (int k = 0; k < NV; ++k) {
-            const int64_t vi = vbeg + t + (int64_t)k * T;
-            if (vi < vend) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&sm.full[s], 1);
+            mbar_init(&sm.empty[s], T / 32);
         }
-        if (crank == 0 && t == 0) {
-            write_masked_outputs(a, row);
-            if (bad) flag_status(a.status, LEAP_DEV_BAD_ID);
+        mbar_init(&sm.ex[0], C);
+        mbar_init(&sm.ex[1], C);
+        sm.abort_flag = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (C > 1) {  // every CTA's barriers are initialised before any remote arrive
+        cluster_arrive_release();
+        cluster_wait_acquire();
+    }
+
+    if (t >= T) {
+        // ---------------- producer warp ----------------
+        const int lane = t - T;
+        uint32_t j = 0;
+        for (int64_t k0 = 0; cid + k0 * ncl < a.N; k0 += 32) {
+            const int64_t row = cid + (k0 + lane) * ncl;
+            bool live = false;
+            int id = 0;
+            if (row < a.N) {
+                const float w = a.w[row];
+                id = a.ids[row];
+                live = (w != 0.f) && id >= 0 && id < V;
+            }
+            uint32_t mask = __ballot_sync(0xffffffffu, live);
+            while (mask) {
+                const int b = __ffs(mask) - 1;
+                mask &= mask - 1;
+                const int idb = __shfl_sync(0xffffffffu, id, b);
+                if (lane == 0) {
+                    const int64_t r = cid + (k0 + b) * ncl;
+                    const uint32_t s = j % STAGES;
+                    if (j >= STAGES) mbar_wait(&sm.empty[s], ((j / STAGES) - 1) & 1u, a.status, &sm.abort_flag);
+                    mbar_arrive_expect_tx(&sm.full[s], nvec * 16u + 16u);
+                    const uint16_t* zr = a.logits + r * a.ld;
+                    if (nvec) bulk_g2s(stage_mem + (size_t)s * per, zr + vbeg * 8, nvec * 16u, &sm.full[s]);
+                    bulk_g2s(&sm.yvec[s], zr + (idb & ~7), 16u, &sm.full[s]);
+                }
+                ++j;
+            }
         }
         return;
     }
 
-    const uint16_t* zr = a.logits + row * a.ld;
-    float zy = 0.f;
-    if (t == 0) zy = bf16_at(zr + id);
-    const uint4* zrow = reinterpret_cast<const uint4*>(zr);
-    uint4 x[NV];
-#pragma unroll
-    for (int k = 0; k < NV; ++k) {
-        const int64_t vi = vbeg + t + (int64_t)k * T;
-        x[k] = (vi < vend) ? ld_stream(zrow + vi) : neg_inf4();
-        if (tailn && vi == V8 - 1) mask_tail(x[k], tailn);
-    }
-    uint32_t mx = kNegInfBf16x2;
-#pragma unroll
-    for (int k = 0; k < NV; ++k) mx = max8(x[k], mx);
-    float m = fmaxf(bf16_lo(mx), bf16_hi(mx));
+    // ---------------- consumers ----------------
+    const int lane = t & 31, warp = t >> 5;
     const float c1 = a.inv_temp * kLog2e;
-    float s = 0.f;
-    if (m != -INFINITY) {
-        const float mc = m * c1;
-        float s0 = 0.f, s1 = 0.f;
-#pragma unroll
-        for (int k = 0; k < NV; k += 2) {
-            s0 += exp_sum8(x[k], c1, mc);
-            if (k + 1 < NV) s1 += exp_sum8(x[k + 1], c1, mc);
+    uint32_t j = 0;
+    float w_next = 0.f;
+    int id_next = 0;
+    if (cid < a.N) {
+        w_next = a.w[cid];
+        id_next = a.ids[cid];
+    }
+    for (int64_t row = cid; row < a.N; row += ncl) {
+        const float wk = w_next;
+        const int id = id_next;
+        if (row + ncl < a.N) {  // next row's scalars, one row ahead
+            w_next = a.w[row + ncl];
+            id_next = a.ids[row + ncl];
         }
-        s = s0 + s1;
-    }
-    warp_lse_merge(m, s, c1);
-    if (lane == 0) wpart[warp] = make_float2(m, s);
-    __syncthreads();
-    if (warp == 0) {
-        const float2 p = (lane < T / 32) ? wpart[lane] : make_float2(-INFINITY, 0.f);
-        m = p.x;
-        s = p.y;
-        warp_lse_merge(m, s, c1);
-        if (lane == 0) cta_part = make_float2(m, s);
-    }
-    if (C > 1) {
-        cluster_arrive_release();
-        cluster_wait_acquire();  // every CTA's cta_part is visible
+        const bool bad = (wk != 0.f) && (id < 0 || id >= V);
+        uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
+        if (wk == 0.f || bad) {  // masked row: same branch in every CTA of the cluster
+#pragma unroll
+            for (int k = 0; k < NV; ++k) {
+                const int64_t vi = vbeg + t + (int64_t)k * T;
+                if (vi < vend) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
+            }
+            if (crank == 0 && t == 0) {
+                write_masked_outputs(a, row);
+                if (bad) flag_status(a.status, LEAP_DEV_BAD_ID);
+            }
+            continue;
+        }
+        float old = 0.f, A = 0.f;
+        if (t == 0) {
+            old = a.old_logp[row];
+            A = a.adv[row];
+        }
+        const uint32_t s = j % STAGES;
+        mbar_wait(&sm.full[s], (j / STAGES) & 1u, a.status, &sm.abort_flag);
+        const uint4* st = stage_mem + (size_t)s * per;
+        uint4 x[NV];
+#pragma unroll
+        for (int k = 0; k < NV; ++k) {
+            const uint32_t li = (uint32_t)(t + k * T);
+            x[k] = (li < nvec) ? st[li] : neg_inf4();
+            if (tailn && vbeg + (int64_t)li == V8 - 1) mask_tail(x[k], tailn);
+        }
+        float zy = 0.f;
+        if (t == 0) zy = bf16_at(reinterpret_cast<const uint16_t*>(&sm.yvec[s]) + (id & 7));
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.empty[s]);  // this warp is done with the stage
+
+        uint32_t mx = kNegInfBf16x2;
+#pragma unroll
+        for (int k = 0; k < NV; ++k) mx = max8(x[k], mx);
+        float m = fmaxf(bf16_lo(mx), bf16_hi(mx));
+        float ssum = 0.f;
+        if (m != -INFINITY) {
+            const float mc = m * c1;
+            float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+            for (int k = 0; k < NV; k += 2) {
+                s0 += exp_sum8(x[k], c1, mc);
+                if (k + 1 < NV) s1 += exp_sum8(x[k + 1], c1, mc);
+            }
+            ssum = s0 + s1;
+        }
+        warp_lse_merge(m, ssum, c1);
+        if (lane == 0) sm.wpart[warp] = make_float2(m, ssum);
+        named_bar_sync(1, T);
         if (warp == 0) {
-            const float2 p = (lane < C) ? ld_cluster_f32x2(cluster_map(smem_addr(&cta_part), (uint32_t)lane))
-                                        : make_float2(-INFINITY, 0.f);
+            const float2 p = (lane < T / 32) ? sm.wpart[lane] : make_float2(-INFINITY, 0.f);
             m = p.x;
-            s = p.y;
-            warp_lse_merge(m, s, c1);
+            ssum = p.y;
+            warp_lse_merge(m, ssum, c1);
+            if (C > 1) {
+                const uint32_t e = j & 1u;
+                if (lane < C) {
+                    st_cluster_f32x2(cluster_map(smem_addr(&sm.slot[e][crank]), (uint32_t)lane), m, ssum);
+                    mbar_arrive_remote(cluster_map(smem_addr(&sm.ex[e]), (uint32_t)lane));
+                }
+                mbar_wait_cluster(&sm.ex[e], (j >> 1) & 1u, a.status, &sm.abort_flag);
+                const volatile float2* sl = &sm.slot[e][0];
+                float2 q = make_float2(-INFINITY, 0.f);
+                if (lane < C) {
+                    q.x = sl[lane].x;
+                    q.y = sl[lane].y;
+                }
+                m = q.x;
+                ssum = q.y;
+                warp_lse_merge(m, ssum, c1);
+            }
+            if (lane == 0) {
+                const TokenLoss r = token_loss(a, m, ssum, zy, old, A, wk);
+                sm.bc[0] = fmaf(m, c1, log2f(ssum));            // log2 of the softmax denominator
+                sm.bc[1] = a.grad_scale * r.g * a.inv_temp;     // dlogits scale
+                if (crank == 0) write_row_outputs(a, row, r, wk);
+            }
         }
-        cluster_arrive_release();  // this CTA is done reading its peers' shared memory
-    }
-    if (t == 0) {
-        const TokenLoss r = token_loss(a, m, s, zy, a.old_logp[row], a.adv[row], wk);
-        bc[0] = fmaf(m, c1, log2f(s));               // log2 of the softmax denominator
-        bc[1] = a.grad_scale * r.g * a.inv_temp;      // dlogits scale
-        if (crank == 0) write_row_outputs(a, row, r, wk);
-    }
-    __syncthreads();
-    const float K = bc[0], coef = bc[1];
-    const int64_t yv = id >> 3;
-    const int ylane = id & 7;
+        named_bar_sync(1, T);
+        const float K = sm.bc[0], coef = sm.bc[1];
+        const int64_t yv = id >> 3;
+        const int ylane = id & 7;
 #pragma unroll
-    for (int k = 0; k < NV; ++k) {
-        const int64_t vi = vbeg + t + (int64_t)k * T;
-        if (vi < vend) {
-            const uint4 d = (coef == 0.f) ? make_uint4(0, 0, 0, 0)
-                                          : dlogit8(x[k], c1, K, coef, vi == yv ? ylane : -1);
-            store_vec(drow, vi, d, V8, tailn);
+        for (int k = 0; k < NV; ++k) {
+            const int64_t vi = vbeg + t + (int64_t)k * T;
+            if (vi < vend) {
+                const uint4 d = (coef == 0.f) ? make_uint4(0, 0, 0, 0)
+                                              : dlogit8(x[k], c1, K, coef, vi == yv ? ylane : -1);
+                store_vec(drow, vi, d, V8, tailn);
+            }
         }
+        ++j;
     }
-    if (C > 1) cluster_wait_acquire();  // peers finished reading cta_part
 }
 
 // ---------------------------------------------------------------------------
@@ -457,30 +555,65 @@ __global__ void __launch_bounds__(kRedThreads) reduce_final_kernel(LossWorkspace
 
 // ---- fused-kernel configurations ------------------------------------------
 struct FusedCfg {
-    int C, T, NV;
+    int C, T, NV, STAGES;
 };
 constexpr FusedCfg kFused[] = {
-    {1, 128, 1}, {1, 256, 4}, {1, 512, 8}, {4, 512, 8}, {8, 256, 10}, {8, 512, 8}, {8, 512, 16},
+    {1, 128, 1, 4}, {1, 256, 4, 3}, {2, 256, 8, 2}, {4, 256, 10, 2}, {8, 256, 10, 2}, {8, 256, 16, 2},
 };
 
-template <int C, int T, int NV>
+template <int C, int T, int NV, int STAGES>
 cudaError_t launch_fused_cfg(const RowArgs& a, cudaStream_t s) {
-    auto kern = fused_loss_kernel<C, T, NV>;
+    auto kern = fused_loss_kernel<C, T, NV, STAGES>;
+    const int64_t V8 = ((int64_t)a.V + 7) >> 3;
+    const int per = (int)((V8 + C - 1) / C);
+    const size_t dyn = (size_t)STAGES * per * 16;
+    // Resident clusters for this shared-memory size (cached per size).
+    static std::mutex mu;
+    static size_t cached_dyn = 0;
+    static int cached_dev = -1;
+    static int cached_ncl = 0;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(a.N * C), 1, 1);
-    cfg.blockDim = dim3(T, 1, 1);
-    cfg.dynamicSmemBytes = 0;
+    cfg.blockDim = dim3(T + 32, 1, 1);
+    cfg.dynamicSmemBytes = dyn;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
     if (C > 1) {
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = C;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
     }
-    return cudaLaunchKernelEx(&cfg, kern, a);
+    int ncl = 0;
+    {
+        std::lock_guard<std::mutex> lk(mu);
+        if (cached_dyn == dyn && cached_dev == dev) {
+            ncl = cached_ncl;
+        } else {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+            if (e != cudaSuccess) return e;
+            cfg.gridDim = dim3(C, 1, 1);
+            if (C > 1) {
+                e = cudaOccupancyMaxActiveClusters(&ncl, kern, &cfg);
+            } else {
+                int per_sm = 0;
+                e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, T + 32, dyn);
+                ncl = per_sm * device_sm_count();
+            }
+            if (e != cudaSuccess) return e;
+            cached_dyn = dyn;
+            cached_dev = dev;
+            cached_ncl = ncl;
+        }
+    }
+    if (ncl <= 0) return cudaErrorNotSupported;
+    if ((int64_t)ncl > a.N) ncl = (int)a.N;
+    cfg.gridDim = dim3((unsigned)(ncl * C), 1, 1);
+    return cudaLaunchKernelEx(&cfg, kern, a, (int32_t)per, (int32_t)ncl);
 }
 
 }  // namespace
@@ -547,13 +680,12 @@ cudaError_t launch_fused_loss(const RowArgs& a, cudaStream_t s) {
     for (const FusedCfg& c : kFused) {
         const int64_t per = (V8 + c.C - 1) / c.C;
         if (per > (int64_t)c.T * c.NV) continue;
-        if (c.C == 1 && c.T == 128) return launch_fused_cfg<1, 128, 1>(a, s);
-        if (c.C == 1 && c.T == 256) return launch_fused_cfg<1, 256, 4>(a, s);
-        if (c.C == 1 && c.T == 512) return launch_fused_cfg<1, 512, 8>(a, s);
-        if (c.C == 4) return launch_fused_cfg<4, 512, 8>(a, s);
-        if (c.C == 8 && c.T == 256) return launch_fused_cfg<8, 256, 10>(a, s);
-        if (c.C == 8 && c.NV == 8) return launch_fused_cfg<8, 512, 8>(a, s);
-        return launch_fused_cfg<8, 512, 16>(a, s);
+        if (c.C == 1 && c.T == 128) return launch_fused_cfg<1, 128, 1, 4>(a, s);
+        if (c.C == 1) return launch_fused_cfg<1, 256, 4, 3>(a, s);
+        if (c.C == 2) return launch_fused_cfg<2, 256, 8, 2>(a, s);
+        if (c.C == 4) return launch_fused_cfg<4, 256, 10, 2>(a, s);
+        if (c.NV == 10) return launch_fused_cfg<8, 256, 10, 2>(a, s);
+        return launch_fused_cfg<8, 256, 16, 2>(a, s);
     }
     return cudaErrorNotSupported;
 }

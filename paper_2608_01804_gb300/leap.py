@@ -26,6 +26,7 @@ LEAP_ERR_BAD_INDEX = 5
 LEAP_DEV_BAD_ID = 1
 LEAP_DEV_BAD_OUTCOME = 2
 LEAP_DEV_BAD_SEGMENT = 4
+LEAP_DEV_TIMEOUT = 8
 
 LEAP_CMP_PAPER = 0
 LEAP_CMP_LEXI = 1

@@ -44,11 +44,12 @@ def _check_rows(out, orc, rows, V, dl=None):
 
 
 @pytest.mark.parametrize("V,ld", [(1024, 1024), (1000, 1008), (1027, 1032), (5000, 5000), (8192, 8192),
-                                  (30001, 30008), (100000, 100000), (151936, 151936), (151936, 152000),
+                                  (30001, 30008), (60000, 60000), (100000, 100000), (151936, 151936), (151936, 152000),
                                   (200000, 200000)])
 def test_fused_loss_all_rows(V, ld):
-    """Every fused configuration (cluster sizes 1, 4, 8), ragged V and padded ld."""
+    """Every fused configuration (cluster sizes 1, 2, 4, 8), ragged V and padded ld."""
     L = leap()
+    L.leap_get_device_status()
     N = 64 if V > 50000 else 256
     z, ids, old, adv, w = _inputs(N, V, seed=V % 97, sigma=3.0, spikes=0.01, ld=ld, old_sigma=0.3)
     ids[:4] = torch.tensor([0, V - 1, min(7, V - 1), min(8, V - 1)], dtype=torch.int32, device="cuda")
@@ -58,6 +59,7 @@ def test_fused_loss_all_rows(V, ld):
     out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, dlogits=torch.full_like(z, 3.0) if ld > V else None)
     if ld > V:
         assert torch.equal(out["dlogits"][:, V:], sentinel)   # columns >= V untouched
+    assert L.leap_get_device_status() == 0              # no bounded wait gave up
     rows = list(range(N))
     orc = _oracle_rows(z, ids, old, adv, w, rows, V)
     _check_rows(out, orc, rows, V, dl=out["dlogits"])

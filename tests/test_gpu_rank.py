@@ -32,8 +32,10 @@ def _compare(gpu, orc, M, strict_A=True):
     assert np.max(np.abs(A - orc["A"].reshape(-1))) <= TOL_ADV
     ta = gpu["turn_adv"].cpu().numpy().astype(np.float64).reshape(n, M)
     assert np.max(np.abs(ta - orc["turn_adv"].reshape(n, M))) <= TOL_ADV
-    # Signs decide the discount base: they must agree exactly where A != 0.
-    nz = orc["A"].reshape(-1) != 0
+    # Signs decide the discount base: they must agree wherever the net score is
+    # nonzero (there |A| >= 1/((G-1)(std+eps)); a zero net score leaves only
+    # rounding noise of the oracle's fp64 mean).
+    nz = np.abs(orc["A"].reshape(-1)) > 1e-9
     assert np.all(np.sign(A[nz]) == np.sign(orc["A"].reshape(-1)[nz]))
 
 
