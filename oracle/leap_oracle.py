@@ -103,7 +103,10 @@ def grpo_advantage(R, eps_std=1e-6, norm=ADVNORM_GRPO_STD, std_unbiased=True):
     """Sec. 3.2, last step: the final advantage A_i by "the standard GRPO formulation".
 
     Reading: A_i = (R_i - mean_g R) / (std_g R + eps_std) over the rollout group,
-    std with the (G - 1) divisor by default.  ``ADVNORM_NONE`` returns R as is.
+    std with the (G - 1) divisor by default.  A group whose rewards are all
+    equal (std = 0) carries no preference signal: its advantages are 0, also
+    when eps_std = 0 (where the formula would read 0/0).  ``ADVNORM_NONE``
+    returns R as is.
     """
     R = np.asarray(R, dtype=np.float64)
     if norm == ADVNORM_NONE:
@@ -113,7 +116,8 @@ def grpo_advantage(R, eps_std=1e-6, norm=ADVNORM_GRPO_STD, std_unbiased=True):
     dev = R - mean
     ddof = 1 if std_unbiased else 0
     std = np.sqrt((dev * dev).sum(axis=1, keepdims=True) / (G - ddof))
-    return dev / (std + eps_std)
+    flat = np.all(R == R[:, :1], axis=1, keepdims=True)
+    return np.where(flat, 0.0, dev / np.where(flat, 1.0, std + eps_std))
 
 
 def turn_advantages(A, T_eff, gamma, M):

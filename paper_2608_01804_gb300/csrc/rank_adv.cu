@@ -103,8 +103,8 @@ __global__ void __launch_bounds__(256) rank_adv_kernel(RankArgs a) {
     // std = sqrt(sum d^2 / (G - 1)^2 / den), den = G - 1 (unbiased) or G.
     const float gm1 = (float)(G - 1);
     float inv_scale;
-    if (a.norm == 1) {
-        inv_scale = 0.f;  // unused
+    if (a.norm == 1 || dd == 0) {
+        inv_scale = 0.f;  // unused, or an all-tied group: no preference signal, A = 0
     } else {
         const double den = a.std_unbiased ? (double)(G - 1) : (double)G;
         const double stdv = sqrt((double)dd / ((double)(G - 1) * (double)(G - 1) * den));

@@ -98,8 +98,9 @@ def test_reward_zero_sum_and_all_tied():
     np.testing.assert_array_equal((nw - nb).sum(axis=1), 0)
     for M in (1, 2, 3):
         for k in range(M + 1):
-            out = _run(_tiers_to_pass_turn([k] * 6, M), M)
-            assert np.all(out["R"] == 0.0) and np.all(out["A"] == 0.0)
+            for eps in (1e-6, 0.0):
+                out = _run(_tiers_to_pass_turn([k] * 6, M), M, eps_std=eps)
+                assert np.all(out["R"] == 0.0) and np.all(out["A"] == 0.0)
 
 
 def test_regime_laws_of_the_intermediate_tier():
