@@ -40,10 +40,6 @@ __device__ __forceinline__ void mask_tail(uint4& x, int n) {
     x = make_uint4(w[0], w[1], w[2], w[3]);
 }
 
-__device__ __forceinline__ uint32_t max8(const uint4& x, uint32_t m) {
-    return max_bf16x2(max_bf16x2(m, x.x), max_bf16x2(max_bf16x2(x.y, x.z), x.w));
-}
-
 // Stores vector vi of a dlogits row; the row's last vector keeps columns >= V intact.
 __device__ __forceinline__ void store_vec(uint4* drow, int64_t vi, uint4 val, int64_t V8, int tailn) {
     if (tailn == 0 || vi != V8 - 1) {
@@ -61,16 +57,38 @@ __device__ __forceinline__ float bf16_at(const uint16_t* p) {
     return __uint_as_float(((uint32_t)*p) << 16);
 }
 
-// sum over the 8 elements of 2^(z * c1 - mc)
-__device__ __forceinline__ float exp_sum8(const uint4& x, float c1, float mc) {
-    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
-    float a0 = 0.f, a1 = 0.f;
+// Max of NV vectors of 8 bf16 as a balanced tree of packed maxima (depth
+// 2 + log2 NV instead of a 4 NV-long chain).
+template <int NV>
+__device__ __forceinline__ float tree_max(const uint4 (&x)[NV]) {
+    uint32_t v[NV];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        a0 += ex2(fmaf(bf16_lo(w[q]), c1, -mc));
-        a1 += ex2(fmaf(bf16_hi(w[q]), c1, -mc));
+    for (int k = 0; k < NV; ++k) v[k] = max_bf16x2(max_bf16x2(x[k].x, x[k].y), max_bf16x2(x[k].z, x[k].w));
+#pragma unroll
+    for (int stride = 1; stride < NV; stride *= 2) {
+#pragma unroll
+        for (int k = 0; k + stride < NV; k += 2 * stride) v[k] = max_bf16x2(v[k], v[k + stride]);
     }
-    return a0 + a1;
+    return fmaxf(bf16_lo(v[0]), bf16_hi(v[0]));
+}
+
+// Sum over NV vectors of 2^(z * c1 - mc), one accumulator per element
+// position (8 independent chains of length NV), then a tree.
+template <int NV>
+__device__ __forceinline__ float tree_exp_sum(const uint4 (&x)[NV], float c1, float mc) {
+    float acc[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[j] = 0.f;
+#pragma unroll
+    for (int k = 0; k < NV; ++k) {
+        const uint32_t w[4] = {x[k].x, x[k].y, x[k].z, x[k].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            acc[2 * q] += ex2(fmaf(bf16_lo(w[q]), c1, -mc));
+            acc[2 * q + 1] += ex2(fmaf(bf16_hi(w[q]), c1, -mc));
+        }
+    }
+    return ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
 }
 
 // dlogits of one vector: coef * (1[v = y] - 2^(z c1 - K)); `yl` is the target's
@@ -172,16 +190,11 @@ __global__ void __launch_bounds__(512) row_stream_kernel(RowArgs a, int mode) {
             x[u] = (vi < V8) ? ld_stream(zrow + vi) : neg_inf4();
             if (tailn && vi == V8 - 1) mask_tail(x[u], tailn);
         }
-        uint32_t mx = kNegInfBf16x2;
-#pragma unroll
-        for (int u = 0; u < U; ++u) mx = max8(x[u], mx);
-        const float bm = fmaxf(bf16_lo(mx), bf16_hi(mx));
+        const float bm = tree_max(x);
         if (bm == -INFINITY) continue;
         const float mn = fmaxf(m, bm);
         const float mc = mn * c1;
-        float acc = 0.f;
-#pragma unroll
-        for (int u = 0; u < U; ++u) acc += exp_sum8(x[u], c1, mc);
+        const float acc = tree_exp_sum(x, c1, mc);
         s = (s == 0.f) ? acc : fmaf(s, ex2((m - mn) * c1), acc);
         m = mn;
     }
@@ -241,8 +254,8 @@ struct FusedSmem {
     int abort_flag;          // set once a bounded wait of this CTA gave up
 };
 
-template <int C, int T, int NV, int STAGES>
-__global__ void __launch_bounds__(T + 32) fused_loss_kernel(RowArgs a, int32_t per, int32_t ncl) {
+template <int C, int T, int NV, int STAGES, int MINB>
+__global__ void __launch_bounds__(T + 32, MINB) fused_loss_kernel(RowArgs a, int32_t per, int32_t ncl) {
     extern __shared__ __align__(128) uint4 stage_mem[];  // STAGES * per vectors
     __shared__ __align__(16) FusedSmem<STAGES, C> sm;
     const int t = threadIdx.x;
@@ -356,21 +369,8 @@ __global__ void __launch_bounds__(T + 32) fused_loss_kernel(RowArgs a, int32_t p
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.empty[s]);  // this warp is done with the stage
 
-        uint32_t mx = kNegInfBf16x2;
-#pragma unroll
-        for (int k = 0; k < NV; ++k) mx = max8(x[k], mx);
-        float m = fmaxf(bf16_lo(mx), bf16_hi(mx));
-        float ssum = 0.f;
-        if (m != -INFINITY) {
-            const float mc = m * c1;
-            float s0 = 0.f, s1 = 0.f;
-#pragma unroll
-            for (int k = 0; k < NV; k += 2) {
-                s0 += exp_sum8(x[k], c1, mc);
-                if (k + 1 < NV) s1 += exp_sum8(x[k + 1], c1, mc);
-            }
-            ssum = s0 + s1;
-        }
+        float m = tree_max(x);
+        float ssum = (m != -INFINITY) ? tree_exp_sum(x, c1, m * c1) : 0.f;
         warp_lse_merge(m, ssum, c1);
         if (lane == 0) sm.wpart[warp] = make_float2(m, ssum);
         named_bar_sync(1, T);
@@ -557,13 +557,23 @@ __global__ void __launch_bounds__(kRedThreads) reduce_final_kernel(LossWorkspace
 struct FusedCfg {
     int C, T, NV, STAGES;
 };
+// The V = 151,936 configuration: shared-memory stages per CTA and the CTAs per
+// SM the register budget is sized for.
+#ifndef LEAP_FUSED_BIG_STAGES
+#define LEAP_FUSED_BIG_STAGES 1
+#endif
+#ifndef LEAP_FUSED_BIG_MINB
+#define LEAP_FUSED_BIG_MINB 3
+#endif
+constexpr int kBigStages = LEAP_FUSED_BIG_STAGES;
+constexpr int kBigMinBlocks = LEAP_FUSED_BIG_MINB;
 constexpr FusedCfg kFused[] = {
     {1, 128, 1, 4}, {1, 256, 4, 3}, {2, 256, 8, 2}, {4, 256, 10, 2}, {8, 256, 10, 2}, {8, 256, 16, 2},
 };
 
-template <int C, int T, int NV, int STAGES>
+template <int C, int T, int NV, int STAGES, int MINB = 1>
 cudaError_t launch_fused_cfg(const RowArgs& a, cudaStream_t s) {
-    auto kern = fused_loss_kernel<C, T, NV, STAGES>;
+    auto kern = fused_loss_kernel<C, T, NV, STAGES, MINB>;
     const int64_t V8 = ((int64_t)a.V + 7) >> 3;
     const int per = (int)((V8 + C - 1) / C);
     const size_t dyn = (size_t)STAGES * per * 16;
@@ -682,9 +692,9 @@ cudaError_t launch_fused_loss(const RowArgs& a, cudaStream_t s) {
         if (per > (int64_t)c.T * c.NV) continue;
         if (c.C == 1 && c.T == 128) return launch_fused_cfg<1, 128, 1, 4>(a, s);
         if (c.C == 1) return launch_fused_cfg<1, 256, 4, 3>(a, s);
-        if (c.C == 2) return launch_fused_cfg<2, 256, 8, 2>(a, s);
-        if (c.C == 4) return launch_fused_cfg<4, 256, 10, 2>(a, s);
-        if (c.NV == 10) return launch_fused_cfg<8, 256, 10, 2>(a, s);
+        if (c.C == 2) return launch_fused_cfg<2, 256, 8, 2, 2>(a, s);
+        if (c.C == 4) return launch_fused_cfg<4, 256, 10, 2, 2>(a, s);
+        if (c.NV == 10) return launch_fused_cfg<8, 256, 10, kBigStages, kBigMinBlocks>(a, s);
         return launch_fused_cfg<8, 256, 16, 2>(a, s);
     }
     return cudaErrorNotSupported;
