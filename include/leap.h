@@ -246,6 +246,37 @@ leap_status_t leap_grpo_loss_fwd(
     void* stream);
 
 /*
+ * leap_grpo_loss_fwd without a workspace argument, for callers that cannot
+ * allocate device memory where they call the loss: a C program that links
+ * only libleap and has no device allocator of its own, or a process whose
+ * device memory is carved up front by a pool that forbids further
+ * cudaMalloc.  The paper has no counterpart; this is an interface variant.
+ * Same arguments and results as leap_grpo_loss_fwd, minus workspace/ws_bytes.
+ * Its scratch is a file-scope device array of 1 MiB, enough for
+ * N <= LEAP_NOALLOC_MAX_ROWS rows; larger N returns LEAP_ERR_INVALID_ARG
+ * (split the batch into chunks and use LEAP_LOSS_ACCUMULATE).  Each device
+ * that loads libleap holds its own copy until the process exits.  The first
+ * call on a device looks the array's device address up (a host-side
+ * cudaGetSymbolAddress with that device current); make that first call
+ * before any stream capture.  Nothing is allocated or freed by any call.
+ * All calls on a device share the one array: calls whose work overlaps on
+ * the GPU (different streams, or host threads) race and give wrong results;
+ * serialise them.  No state carries over between calls: every call writes
+ * all of the scratch it later reads, so nothing needs clearing.
+ */
+#define LEAP_NOALLOC_MAX_ROWS 65536
+
+leap_status_t leap_grpo_loss_fwd_noalloc(
+    const leap_loss_params_t* params,
+    const uint16_t* logits, int64_t ld, const int32_t* ids,
+    const float* old_logp, const float* adv, const float* w,
+    int64_t N, int32_t V,
+    float* loss, float* logp, float* lse, float* ell,
+    uint16_t* dlogits,
+    leap_loss_stats_t* stats,
+    void* stream);
+
+/*
  * Split backward: dlogits from logits and the lse saved by the forward
  * (reads logits once more: 2V bytes read + 2V written per live row).
  * Same argument meanings as leap_grpo_loss_fwd; lse f32 [N] required.

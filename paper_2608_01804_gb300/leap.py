@@ -41,7 +41,9 @@ EXPORTS = (
     "leap_status_string", "leap_version", "leap_get_device_status",
     "leap_group_rank_advantages", "leap_rollout_token_counts", "leap_scatter_turn_advantages",
     "leap_token_logprobs", "leap_grpo_loss_workspace_size", "leap_grpo_loss_fwd", "leap_grpo_loss_bwd",
+    "leap_grpo_loss_fwd_noalloc",
 )
+LEAP_NOALLOC_MAX_ROWS = 65536
 
 
 class LeapError(RuntimeError):
@@ -102,6 +104,9 @@ def lib() -> ctypes.CDLL:
     L.leap_grpo_loss_fwd.restype = S
     L.leap_grpo_loss_fwd.argtypes = [ctypes.POINTER(LossParams), _P, _I64, _P, _P, _P, _P, _I64, _I32,
                                      _P, _P, _P, _P, _P, _P, _SZ, _P, _P]
+    L.leap_grpo_loss_fwd_noalloc.restype = S
+    L.leap_grpo_loss_fwd_noalloc.argtypes = [ctypes.POINTER(LossParams), _P, _I64, _P, _P, _P, _P, _I64, _I32,
+                                             _P, _P, _P, _P, _P, _P, _P]
     L.leap_grpo_loss_bwd.restype = S
     L.leap_grpo_loss_bwd.argtypes = [ctypes.POINTER(LossParams), _P, _I64, _P, _P, _P, _P, _P, _I64, _I32,
                                      _P, _P]
@@ -257,6 +262,31 @@ def leap_grpo_loss_fwd(logits, ids, old_logp, adv, w, *, V=None, eps_low=0.2, ep
                                   None if dlogits is None else ctypes.c_void_p(dlogits.data_ptr()),
                                   _ptr(workspace), workspace.numel(), _ptr(stats), _stream(stream))
     _check(st, "leap_grpo_loss_fwd")
+    return dict(loss=loss, logp=logp, lse=lse, ell=ell, dlogits=dlogits)
+
+
+def leap_grpo_loss_fwd_noalloc(logits, ids, old_logp, adv, w, *, V=None, eps_low=0.2, eps_high=0.2,
+                               inv_temp=1.0, grad_scale=1.0, accumulate=False, loss=None, logp=None, lse=None,
+                               ell=None, dlogits=None, want_dlogits=True, want_outputs=True, stats=None,
+                               stream=None):
+    """leap_grpo_loss_fwd whose scratch is libleap's own device array (no workspace
+    argument, N <= LEAP_NOALLOC_MAX_ROWS).  The output tensors are still the caller's."""
+    lp, ld, V = _logits_args(logits, V)
+    N = logits.shape[0]
+    if loss is None:
+        loss = torch.zeros(1, dtype=torch.float32, device=logits.device)
+    if want_outputs:
+        logp = _empty(N, torch.float32, logits) if logp is None else logp
+        lse = _empty(N, torch.float32, logits) if lse is None else lse
+        ell = _empty(N, torch.float32, logits) if ell is None else ell
+    if dlogits is None and want_dlogits:
+        dlogits = torch.empty_like(logits)
+    p = LossParams(eps_low, eps_high, inv_temp, grad_scale, LEAP_LOSS_ACCUMULATE if accumulate else 0)
+    st = lib().leap_grpo_loss_fwd_noalloc(ctypes.byref(p), lp, ld, _ptr(ids), _ptr(old_logp), _ptr(adv), _ptr(w),
+                                          N, V, _ptr(loss), _ptr(logp), _ptr(lse), _ptr(ell),
+                                          None if dlogits is None else ctypes.c_void_p(dlogits.data_ptr()),
+                                          _ptr(stats), _stream(stream))
+    _check(st, "leap_grpo_loss_fwd_noalloc")
     return dict(loss=loss, logp=logp, lse=lse, ell=ell, dlogits=dlogits)
 
 
