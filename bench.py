@@ -61,6 +61,7 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-rows", action="store_true", help="skip the per-row measurements")
     ap.add_argument("--prompts", type=int, default=16,
                     help="prompts per rank (16 = the benchmark workload; fewer only for profiling captures)")
     return ap.parse_args()
@@ -233,6 +234,99 @@ def reference_arm(args):
     print(json.dumps(line), flush=True)
 
 
+def _timed_launches(fn, reps, stream, flush=None):
+    """Average device time of fn() over `reps` launches, each timed with CUDA
+    events on the launching stream; `flush` (untimed) runs before each."""
+    total = 0.0
+    for _ in range(reps):
+        if flush is not None:
+            flush()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        b.synchronize()
+        total += a.elapsed_time(b)
+    return total / reps
+
+
+def measure_rows(device, logits, ids, old, step, peak, reps=5):
+    """Each remaining row of the hot path on its own workload, against the HBM
+    roofline: rank advantages on 65,536 groups x 64 rollouts (M = 3), token
+    counts + scatter on the packed multi-turn batch, log-probs and the split
+    forward / backward on the single-turn batch."""
+    from paper_2608_01804_gb300 import leap as L
+    from paper_2608_01804_gb300 import synth
+    stream = torch.cuda.current_stream()
+    flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device=device)   # > L2: evicts between launches
+    flush = lambda: flush_buf.fill_(1)
+    rows = {}
+
+    def entry(bytes_, ms, unit_count, unit):
+        gbs = bytes_ / (ms / 1e3) / 1e9
+        return {"ms": ms, "algorithmic_bytes": bytes_, "achieved_gbs": gbs, "frac": gbs / peak,
+                "throughput": unit_count / (ms / 1e3), "unit": unit}
+
+    # a1-a3: rank advantages, tournament stress workload.
+    pt, nt, _, _ = synth.tournament_outcomes()
+    G, M = 64, 3
+    n = pt.size
+    pt_d = torch.as_tensor(pt).to(device)
+    nt_d = torch.as_tensor(nt).to(device)
+    out = L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=50, tau_max=56, gamma=0.9)
+    fn = lambda: L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=50, tau_max=56, gamma=0.9, out=out)
+    fn()
+    ms = _timed_launches(fn, reps * 4, stream, flush)
+    rank_bytes = n * (2 + 1 + 4 + 4 + 4 + 4 + 4 * M + 1) + n // G
+    rows["rank_advantages_65536x64"] = entry(rank_bytes, ms, n, "rollouts/s")
+    del pt_d, nt_d, out
+
+    # a4: per-rollout counts + per-token scatter, packed multi-turn batch.
+    b = synth.multiturn_dcp_batch()
+    pt_d = torch.as_tensor(b.pass_turn).to(device)
+    nt_d = torch.as_tensor(b.num_turns).to(device)
+    rk = L.leap_group_rank_advantages(pt_d, nt_d, G=b.G, M=b.M, tau_min=8, tau_max=15, gamma=0.9)
+    so = torch.as_tensor(b.seg_offsets).to(device)
+    sr = torch.as_tensor(b.seg_rollout).to(device)
+    st_ = torch.as_tensor(b.seg_turn).to(device)
+    Lc, tot = L.leap_rollout_token_counts(b.N, so, sr, st_, rk["T_eff"], M=b.M)
+    adv, w = L.leap_scatter_turn_advantages(b.N, so, sr, st_, rk["turn_adv"], rk["T_eff"], Lc, tot, M=b.M)
+
+    def tok():
+        L.leap_rollout_token_counts(b.N, so, sr, st_, rk["T_eff"], M=b.M, L=Lc, totals=tot)
+        L.leap_scatter_turn_advantages(b.N, so, sr, st_, rk["turn_adv"], rk["T_eff"], Lc, tot, M=b.M, adv=adv, w=w)
+    ms = _timed_launches(tok, reps * 4, stream, flush)
+    rows["token_counts_scatter_multiturn_%d_tokens" % b.N] = entry(8 * b.N, ms, b.N, "tokens/s")
+    del adv, w
+
+    # a5: log-probs (2V bytes per row), and the split forward / backward (a6, a7).
+    N = logits.shape[0]
+    logp = torch.empty(N, dtype=torch.float32, device=device)
+    lse = torch.empty(N, dtype=torch.float32, device=device)
+    fn = lambda: L.leap_token_logprobs(logits, ids, V=V, logp=logp, lse=lse)
+    fn()
+    ms = _timed_launches(fn, reps, stream)
+    rows["token_logprobs_32768xV"] = entry(2 * V * N + 12 * N, ms, N, "tokens/s")
+    live = int((step.w != 0).sum().item())
+    ws = L.loss_workspace(N, V, device)
+    fwd = lambda: L.leap_grpo_loss_fwd(logits, ids, old, step.adv, step.w, V=V, loss=step.loss, lse=lse,
+                                       want_dlogits=False, want_outputs=False, workspace=ws)
+    fwd()
+    ms_f = _timed_launches(fwd, reps, stream)
+    rows["loss_fwd_only_32768xV"] = entry(2 * V * live + 16 * N, ms_f, live, "valid tokens/s")
+    dl = torch.empty_like(logits)
+    bwd = lambda: L.leap_grpo_loss_bwd(logits, ids, old, step.adv, step.w, lse, V=V, dlogits=dl)
+    bwd()
+    ms_b = _timed_launches(bwd, reps, stream)
+    rows["loss_bwd_split_32768xV"] = entry(4 * V * live + 2 * V * (N - live) + 20 * N, ms_b, live, "valid tokens/s")
+    split = entry(6 * V * live + 2 * V * (N - live) + 36 * N, ms_f + ms_b, live, "valid tokens/s")
+    split["frac_vs_fused_4V_bytes"] = (4 * V * live + 2 * V * (N - live) + 16 * N) / ((ms_f + ms_b) / 1e3) / 1e9 / peak
+    rows["split_fwd_then_bwd_32768xV"] = split
+    del dl, ws, flush_buf
+    torch.cuda.synchronize()
+    return rows
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -346,12 +440,16 @@ def main():
                "d2h_bytes_per_step": 4, "ms_per_step": e_ms, "steps": E}
         del host
 
+    rows = None
+    if rank == 0 and not args.no_rows and args.prompts == 16:
+        rows = measure_rows(device, logits, ids, old, step, peak)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rate, rows, valid, secs = cpu_oracle_rate(batch, logits, ids, old, args.cpu_seconds)
+        rate, n_rows, valid, secs = cpu_oracle_rate(batch, logits, ids, old, args.cpu_seconds)
         cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": "rank/token oracle on the whole batch + loss fwd and dlogits on the first %d rows "
-                         "(%d valid tokens), %.1f s of CPU time" % (rows, valid, secs)}
+                         "(%d valid tokens), %.1f s of CPU time" % (n_rows, valid, secs)}
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
@@ -361,7 +459,7 @@ def main():
                            "rows_per_step_per_gpu": N, "valid_tokens_per_step_per_gpu": n_valid,
                            "vocab": V, "logits_dtype": "bf16", "l2": "inputs larger than L2 (9.96 GB of logits "
                            "read and 9.96 GB of dlogits written per step)", "parallelism": "dp%d" % world},
-                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+                "roofline": roofline, "rows": rows, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": K * GrpoStep.LAUNCHES_PER_RUN, "clocks": clk}
         print(json.dumps(line), flush=True)
     if pg is not None:
