@@ -156,8 +156,8 @@ __device__ __forceinline__ void write_masked_outputs(const RowArgs& a, int64_t r
 // 512: one row per CTA), U vectors of 8 bf16 in flight per thread.
 // mode 0: log-probs (every row read); mode 1: loss forward (w == 0 rows skipped).
 // ---------------------------------------------------------------------------
-template <int TPR, int U>
-__global__ void __launch_bounds__(512) row_stream_kernel(RowArgs a, int mode) {
+template <int TPR, int U, int MINB>
+__global__ void __launch_bounds__(512, MINB) row_stream_kernel(RowArgs a, int mode) {
     __shared__ float2 wpart[16];
     const int t = threadIdx.x % TPR;
     const int64_t row = (int64_t)blockIdx.x * (blockDim.x / TPR) + threadIdx.x / TPR;
@@ -665,9 +665,9 @@ cudaError_t launch_row_stream(const RowArgs& a, int mode, cudaStream_t s) {
     const int64_t V8 = ((int64_t)a.V + 7) >> 3;
     if (V8 <= 128) {
         const int64_t blocks = (a.N + 7) / 8;
-        row_stream_kernel<32, 4><<<(unsigned)blocks, 256, 0, s>>>(a, mode);
+        row_stream_kernel<32, 4, 1><<<(unsigned)blocks, 256, 0, s>>>(a, mode);
     } else {
-        row_stream_kernel<512, 8><<<(unsigned)a.N, 512, 0, s>>>(a, mode);
+        row_stream_kernel<512, 4, 3><<<(unsigned)a.N, 512, 0, s>>>(a, mode);
     }
     return cudaGetLastError();
 }

@@ -100,15 +100,15 @@ __global__ void __launch_bounds__(256) rank_adv_kernel(RankArgs a) {
 
     // GRPO standardisation.  mean_g R = 0 exactly (every strict pair adds +1
     // and -1 to the net scores), so A_i = d_i / ((G - 1) (std + eps)) with
-    // std = sqrt(sum d^2 / (G - 1)^2 / den), den = G - 1 (unbiased) or G.
+    // (G - 1) std = sqrt(sum d^2 / den), den = G - 1 (unbiased) or G.  fp32
+    // with IEEE division and square root: at most ~3.5 ulp on A.
     const float gm1 = (float)(G - 1);
     float inv_scale;
     if (a.norm == 1 || dd == 0) {
         inv_scale = 0.f;  // unused, or an all-tied group: no preference signal, A = 0
     } else {
-        const double den = a.std_unbiased ? (double)(G - 1) : (double)G;
-        const double stdv = sqrt((double)dd / ((double)(G - 1) * (double)(G - 1) * den));
-        inv_scale = (float)(1.0 / ((double)(G - 1) * (stdv + (double)a.eps_std)));
+        const float den = a.std_unbiased ? gm1 : (float)G;
+        inv_scale = 1.f / (sqrtf((float)dd / den) + gm1 * a.eps_std);
     }
 #pragma unroll
     for (int j = 0; j < J; ++j) {
@@ -200,32 +200,58 @@ __global__ void totals_kernel(const int32_t* L, int32_t n, int64_t* totals) {
 
 // ---- per-token scatter ------------------------------------------------------
 
-__global__ void scatter_kernel(SegArgs a) {
+// 1 / x for an exact positive integer x, as fp32 rounded once: IEEE fp32
+// division when x fits the 24-bit significand, else fp64 then rounding.
+__device__ __forceinline__ float recip_count(double x) {
+    return (x < 16777216.0) ? 1.f / (float)x : (float)(1.0 / x);
+}
+
+// One warp per chunk of 32 * kScatterIters consecutive tokens: lane 0 finds
+// the chunk's first segment by binary search, then every lane walks forward
+// through the (non-decreasing) offsets as its tokens advance.
+constexpr int kScatterIters = 8;
+
+__global__ void __launch_bounds__(256) scatter_kernel(SegArgs a) {
     const int64_t nv = a.totals_in[0];
     const int64_t rv = a.totals_in[1];
     const int32_t S = a.num_segs;
-    for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < a.N; k += (int64_t)gridDim.x * blockDim.x) {
-        float adv = 0.f, w = 0.f;
-        if (S > 0 && k >= a.seg_offsets[0] && k < a.seg_offsets[S]) {
-            // Last s with seg_offsets[s] <= k (upper bound - 1).
-            int32_t lo = 0, hi = S;  // search in [lo, hi)
+    const int lane = threadIdx.x & 31;
+    const int64_t chunk = (int64_t)32 * kScatterIters;
+    const int64_t nchunks = (a.N + chunk - 1) / chunk;
+    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    for (int64_t c = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); c < nchunks; c += warps) {
+        const int64_t k0 = c * chunk;
+        int32_t seg = 0;
+        if (lane == 0 && S > 0) {  // last s with seg_offsets[s] <= k0 (0 if none)
+            int32_t lo = 0, hi = S;
             while (hi - lo > 1) {
                 const int32_t mid = (lo + hi) >> 1;
-                if (a.seg_offsets[mid] <= k) lo = mid; else hi = mid;
+                if (a.seg_offsets[mid] <= k0) lo = mid; else hi = mid;
             }
-            int32_t a0, b0, i, t;
-            if (segment_ok(a, lo, a0, b0, i, t) && k >= a0 && k < b0 && t >= 0 && t < (int)a.T_eff[i]) {
-                adv = a.turn_adv[(int64_t)i * a.M + t];
-                if (a.agg == 1) {
-                    w = nv > 0 ? (float)(1.0 / (double)nv) : 0.f;
-                } else {
-                    const int32_t L = a.L_in[i];
-                    w = (rv > 0 && L > 0) ? (float)(1.0 / ((double)rv * (double)L)) : 0.f;
+            seg = lo;
+        }
+        seg = __shfl_sync(0xffffffffu, seg, 0);
+#pragma unroll 1
+        for (int it = 0; it < kScatterIters; ++it) {
+            const int64_t k = k0 + it * 32 + lane;
+            if (k >= a.N) break;
+            float adv = 0.f, w = 0.f;
+            if (S > 0) {
+                while (seg + 1 < S && a.seg_offsets[seg + 1] <= k) ++seg;
+                int32_t lo, hi, i, t;
+                if (segment_ok(a, seg, lo, hi, i, t) && k >= lo && k < hi && t >= 0 && t < (int)a.T_eff[i]) {
+                    adv = a.turn_adv[(int64_t)i * a.M + t];
+                    if (a.agg == 1) {
+                        w = nv > 0 ? recip_count((double)nv) : 0.f;
+                    } else {
+                        const int32_t L = a.L_in[i];
+                        w = (rv > 0 && L > 0) ? recip_count((double)rv * (double)L) : 0.f;
+                    }
                 }
             }
+            a.adv_out[k] = adv;
+            a.w_out[k] = w;
         }
-        a.adv_out[k] = adv;
-        a.w_out[k] = w;
     }
 }
 
@@ -258,7 +284,8 @@ cudaError_t launch_token_counts(const SegArgs& a, cudaStream_t s) {
 cudaError_t launch_scatter(const SegArgs& a, cudaStream_t s) {
     if (a.N == 0) return cudaSuccess;
     const int sms = device_sm_count();
-    const int64_t blocks = std::min<int64_t>((a.N + 255) / 256, (int64_t)sms * 8);
+    const int64_t chunks = (a.N + 32 * kScatterIters - 1) / (32 * kScatterIters);
+    const int64_t blocks = std::min<int64_t>((chunks + 7) / 8, (int64_t)sms * 16);
     scatter_kernel<<<(unsigned)blocks, 256, 0, s>>>(a);
     return cudaGetLastError();
 }
