@@ -40,7 +40,7 @@ WORKLOAD = ("single-turn GRPO: 16 prompts x G=8 x 256 token slots = 32,768 rows 
 # dram bytes (read + write) of one fused_loss_kernel launch on this workload: an ncu capture of the
 # kernel built from sources with this SHA-256 on a 4,096-row slice, scaled to the full launch by
 # algorithmic bytes (traffic grows in proportion to them); null once the sources change.
-KNOWN_TRAFFIC = {"src_sha256": "d8a24a07afd04004b371685da3d2c32df955850fb6a255469c17cf0c63eee287", "bytes_per_launch": 16031996848}
+KNOWN_TRAFFIC = {"src_sha256": "719d7f95fc58e9df03814195268dd11a1da3831c83618cee9e3bb9d4593f1fb1", "bytes_per_launch": 16099568938}
 KERNEL_SOURCES = ("paper_2608_01804_gb300/csrc/logprob_loss.cu", "paper_2608_01804_gb300/csrc/leap_common.cuh")
 
 
@@ -400,7 +400,7 @@ def main():
     if KNOWN_TRAFFIC and KNOWN_TRAFFIC.get("src_sha256") == _src_sha():
         traffic = KNOWN_TRAFFIC["bytes_per_launch"]
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                "traffic": traffic, "kernel": "fused_loss_kernel<8,256,10,1,3> (+2 reduce launches in the timing)",
+                "traffic": traffic, "kernel": "fused_loss_l2_kernel<1024,4,1> (+2 reduce launches in the timing)",
                 "algorithmic_bytes_per_launch": alg_bytes, "launch_ms": loss_ms, "peak_source": peak_kind}
 
     # End to end through the same public calls, inputs copied from pinned host memory every step.

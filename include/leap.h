@@ -203,6 +203,12 @@ leap_status_t leap_token_logprobs(
  * logp/lse/ell are written as 0 and their dlogits row as zeros.
  * ------------------------------------------------------------------------ */
 #define LEAP_LOSS_ACCUMULATE 1u  /* loss[0] += this call's sum (chunked passes) */
+/* Fused backward through the cluster kernel: each logits row is split over 8
+ * CTAs that hold it in registers, so it is read from HBM exactly once whatever
+ * else is using L2 (supports V <= 262,144).  The default kernel reads a row
+ * twice, the second time from L2, which is faster when the loss pass has the
+ * GPU's L2 to itself. */
+#define LEAP_LOSS_SINGLE_READ 2u
 
 typedef struct {
     float eps_low;     /* >= 0 */
@@ -231,8 +237,8 @@ size_t leap_grpo_loss_workspace_size(int64_t N, int32_t V);
  * Outputs: loss f32 [1] (required); logp, lse, ell f32 [N] (optional);
  * dlogits bf16 [N x ld] (optional; columns >= V untouched); stats optional.
  * workspace: >= leap_grpo_loss_workspace_size(N, V) bytes, 256-byte aligned,
- * contents ignored on entry.  Requires 1 <= V; the fused backward supports
- * V up to 262,144 (LEAP_ERR_UNSUPPORTED beyond: use the split path).
+ * contents ignored on entry.  Requires 1 <= V.  With LEAP_LOSS_SINGLE_READ
+ * the fused backward supports V up to 262,144 (LEAP_ERR_UNSUPPORTED beyond).
  */
 leap_status_t leap_grpo_loss_fwd(
     const leap_loss_params_t* params,

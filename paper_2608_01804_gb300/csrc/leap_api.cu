@@ -233,7 +233,7 @@ static bool loss_params_ok(const leap_loss_params_t* p) {
     if (!p) return false;
     if (!finite(p->eps_low) || !finite(p->eps_high) || p->eps_low < 0.f || p->eps_high < 0.f) return false;
     if (!finite(p->inv_temp) || !(p->inv_temp > 0.f) || !finite(p->grad_scale)) return false;
-    if (p->flags & ~LEAP_LOSS_ACCUMULATE) return false;
+    if (p->flags & ~(LEAP_LOSS_ACCUMULATE | LEAP_LOSS_SINGLE_READ)) return false;
     return true;
 }
 
@@ -254,7 +254,8 @@ leap_status_t leap_grpo_loss_fwd(const leap_loss_params_t* p, const uint16_t* lo
     if (dlogits && !aligned16(dlogits)) return LEAP_ERR_INVALID_ARG;
     if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return LEAP_ERR_INVALID_ARG;
     if (ws_bytes < loss_workspace_bytes(N)) return LEAP_ERR_INVALID_ARG;
-    if (dlogits && (int64_t)V > fused_max_vocab()) return LEAP_ERR_UNSUPPORTED;
+    const bool single_read = (p->flags & LEAP_LOSS_SINGLE_READ) != 0;
+    if (dlogits && single_read && (int64_t)V > fused_max_vocab()) return LEAP_ERR_UNSUPPORTED;
     const LossWorkspace ws = carve_loss_workspace(workspace, N);
     RowArgs a = {};
     a.logits = logits;
@@ -279,7 +280,7 @@ leap_status_t leap_grpo_loss_fwd(const leap_loss_params_t* p, const uint16_t* lo
     a.status = status_ptr();
     if (!a.status) return LEAP_ERR_CUDA;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    cudaError_t e = dlogits ? launch_fused_loss(a, s) : launch_row_stream(a, 1, s);
+    cudaError_t e = dlogits ? launch_fused_loss(a, single_read, s) : launch_row_stream(a, 1, s);
     if (e != cudaSuccess) return from_cuda(e);
     return from_cuda(launch_loss_reduce(ws, N, loss, stats, (p->flags & LEAP_LOSS_ACCUMULATE) != 0, s));
 }

@@ -89,8 +89,9 @@ cudaError_t launch_scatter(const SegArgs& a, cudaStream_t s);
 
 // mode: 0 = log-probs only, 1 = loss forward (no dlogits).
 cudaError_t launch_row_stream(const RowArgs& a, int mode, cudaStream_t s);
-// Fused forward + backward; returns cudaErrorNotSupported if V is too large.
-cudaError_t launch_fused_loss(const RowArgs& a, cudaStream_t s);
+// Fused forward + backward: the L2 two-pass kernel, or with single_read the
+// cluster-resident one (cudaErrorNotSupported if V is too large for it).
+cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s);
 cudaError_t launch_split_bwd(const RowArgs& a, cudaStream_t s);
 cudaError_t launch_loss_reduce(const LossWorkspace& ws, int64_t N, float* loss, void* stats,
                                bool accumulate, cudaStream_t s);

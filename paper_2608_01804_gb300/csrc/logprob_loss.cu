@@ -5,11 +5,13 @@
 //   row_stream_kernel  one pass over each logits row with an online
 //                      (max, sum) -> log-probs, or the loss forward without
 //                      dlogits.  2V bytes read per row.
-//   fused_loss_kernel  forward + backward in one pass.  A row is split over a
-//                      cluster of C CTAs; each CTA keeps its slice in
-//                      registers, the CTAs exchange one (max, sum) pair
-//                      through distributed shared memory, then each writes
-//                      its dlogits slice.  2V read + 2V written per row.
+//   fused_loss_l2_kernel  forward + backward, one CTA per row, the second pass
+//                      over the row served by L2.  2V read + 2V written per row.
+//   fused_loss_kernel  forward + backward with the row split over a cluster
+//                      of C CTAs that keep their slices in registers and
+//                      exchange one (max, sum) pair through distributed
+//                      shared memory: each row is read from HBM exactly once
+//                      whatever else uses L2 (LEAP_LOSS_SINGLE_READ).
 //   split_bwd_kernel   dlogits from a saved lse: 2V read + 2V written.
 //   reduce kernels     fixed-order fp64 sum of the per-row loss terms.
 #include "../../include/leap.h"
@@ -421,6 +423,104 @@ __global__ void __launch_bounds__(T + 32, MINB) fused_loss_kernel(RowArgs a, int
 }
 
 // ---------------------------------------------------------------------------
+// Fused forward + backward (default): one CTA of T threads per row and at most
+// one resident CTA per SM, two passes over the row.  The first reads it from
+// HBM with an evict_last L2 policy and reduces it; the second reads it back
+// with an evict_first policy and writes dlogits with streaming stores.  With
+// one row per SM in flight (152 rows, 46 MB at V = 151,936) the second read is
+// an L2 hit: DRAM sees 2V bytes read and 2V written per live row.
+// ---------------------------------------------------------------------------
+template <int T, int U, int MINB>
+__global__ void __launch_bounds__(T, MINB) fused_loss_l2_kernel(RowArgs a) {
+    __shared__ float2 wpart[T / 32];
+    __shared__ float bc[2];
+    const int64_t row = blockIdx.x;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int V = a.V;
+    const int64_t V8 = ((int64_t)V + 7) >> 3;
+    const int tailn = V & 7;
+    const float wk = a.w[row];
+    const int id = a.ids[row];
+    const bool bad = (wk != 0.f) && (id < 0 || id >= V);
+    uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
+    if (wk == 0.f || bad) {
+        for (int64_t vi = t; vi < V8; vi += T) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
+        if (t == 0) {
+            write_masked_outputs(a, row);
+            if (bad) flag_status(a.status, LEAP_DEV_BAD_ID);
+        }
+        return;
+    }
+    const uint16_t* zr = a.logits + row * a.ld;
+    const uint4* zrow = reinterpret_cast<const uint4*>(zr);
+    float zy = 0.f, old = 0.f, A = 0.f;
+    if (t == 0) {
+        zy = bf16_at(zr + id);
+        old = a.old_logp[row];
+        A = a.adv[row];
+    }
+    const uint64_t keep = l2_policy_evict_last();
+    const float c1 = a.inv_temp * kLog2e;
+    float m = -INFINITY, s = 0.f;
+    for (int64_t v0 = t; v0 < V8; v0 += (int64_t)T * U) {
+        uint4 x[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t vi = v0 + (int64_t)u * T;
+            x[u] = (vi < V8) ? ld_stream_hint(zrow + vi, keep) : neg_inf4();
+            if (tailn && vi == V8 - 1) mask_tail(x[u], tailn);
+        }
+        const float bm = tree_max(x);
+        if (bm == -INFINITY) continue;
+        const float mn = fmaxf(m, bm);
+        const float acc = tree_exp_sum(x, c1, mn * c1);
+        s = (s == 0.f) ? acc : fmaf(s, ex2((m - mn) * c1), acc);
+        m = mn;
+    }
+    warp_lse_merge(m, s, c1);
+    if (lane == 0) wpart[warp] = make_float2(m, s);
+    __syncthreads();
+    if (warp == 0) {
+        const float2 p = (lane < T / 32) ? wpart[lane] : make_float2(-INFINITY, 0.f);
+        m = p.x;
+        s = p.y;
+        warp_lse_merge(m, s, c1);
+        if (lane == 0) {
+            const TokenLoss r = token_loss(a, m, s, zy, old, A, wk);
+            bc[0] = fmaf(m, c1, log2f(s));
+            bc[1] = a.grad_scale * r.g * a.inv_temp;
+            write_row_outputs(a, row, r, wk);
+        }
+    }
+    __syncthreads();
+    const float K = bc[0], coef = bc[1];
+    const uint64_t drop = l2_policy_evict_first();
+    const int64_t yv = id >> 3;
+    const int ylane = id & 7;
+    for (int64_t v0 = t; v0 < V8; v0 += (int64_t)T * U) {
+        if (coef == 0.f) {
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int64_t vi = v0 + (int64_t)u * T;
+                if (vi < V8) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
+            }
+            continue;
+        }
+        uint4 x[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t vi = v0 + (int64_t)u * T;
+            x[u] = (vi < V8) ? ld_stream_hint(zrow + vi, drop) : neg_inf4();
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t vi = v0 + (int64_t)u * T;
+            if (vi < V8) store_vec(drow, vi, dlogit8(x[u], c1, K, coef, vi == yv ? ylane : -1), V8, tailn);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Split backward from the saved lse.  Every thread recomputes the row's scalar
 // coefficient from broadcast loads, so no block synchronisation is needed.
 // ---------------------------------------------------------------------------
@@ -557,16 +657,10 @@ __global__ void __launch_bounds__(kRedThreads) reduce_final_kernel(LossWorkspace
 struct FusedCfg {
     int C, T, NV, STAGES;
 };
-// The V = 151,936 configuration: shared-memory stages per CTA and the CTAs per
-// SM the register budget is sized for.
-#ifndef LEAP_FUSED_BIG_STAGES
-#define LEAP_FUSED_BIG_STAGES 1
-#endif
-#ifndef LEAP_FUSED_BIG_MINB
-#define LEAP_FUSED_BIG_MINB 3
-#endif
-constexpr int kBigStages = LEAP_FUSED_BIG_STAGES;
-constexpr int kBigMinBlocks = LEAP_FUSED_BIG_MINB;
+// The V = 151,936 configuration: one shared-memory stage per CTA and a
+// register budget for three CTAs per SM (51 resident clusters).
+constexpr int kBigStages = 1;
+constexpr int kBigMinBlocks = 3;
 constexpr FusedCfg kFused[] = {
     {1, 128, 1, 4}, {1, 256, 4, 3}, {2, 256, 8, 2}, {4, 256, 10, 2}, {8, 256, 10, 2}, {8, 256, 16, 2},
 };
@@ -684,8 +778,12 @@ cudaError_t launch_split_bwd(const RowArgs& a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_fused_loss(const RowArgs& a, cudaStream_t s) {
+cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s) {
     if (a.N == 0) return cudaSuccess;
+    if (!single_read) {
+        fused_loss_l2_kernel<1024, 4, 1><<<(unsigned)a.N, 1024, 0, s>>>(a);
+        return cudaGetLastError();
+    }
     const int64_t V8 = ((int64_t)a.V + 7) >> 3;
     for (const FusedCfg& c : kFused) {
         const int64_t per = (V8 + c.C - 1) / c.C;

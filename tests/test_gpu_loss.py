@@ -43,11 +43,13 @@ def _check_rows(out, orc, rows, V, dl=None):
         check_dlogits_rows(bf16_rows_to_f64(dl.index_select(0, sel)[:, :V]), orc, rows)
 
 
+@pytest.mark.parametrize("single_read", [False, True])
 @pytest.mark.parametrize("V,ld", [(1024, 1024), (1000, 1008), (1027, 1032), (5000, 5000), (8192, 8192),
                                   (30001, 30008), (60000, 60000), (100000, 100000), (151936, 151936), (151936, 152000),
                                   (200000, 200000)])
-def test_fused_loss_all_rows(V, ld):
-    """Every fused configuration (cluster sizes 1, 2, 4, 8), ragged V and padded ld."""
+def test_fused_loss_all_rows(V, ld, single_read):
+    """Both fused kernels (the L2 two-pass one, and with single_read every
+    cluster configuration, sizes 1, 2, 4, 8), ragged V and padded ld."""
     L = leap()
     L.leap_get_device_status()
     N = 64 if V > 50000 else 256
@@ -56,7 +58,8 @@ def test_fused_loss_all_rows(V, ld):
     w[:4] = 0.1
     if ld > V:
         sentinel = torch.full((N, ld - V), 3.0, dtype=torch.bfloat16, device="cuda")
-    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, dlogits=torch.full_like(z, 3.0) if ld > V else None)
+    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, dlogits=torch.full_like(z, 3.0) if ld > V else None,
+                               single_read=single_read)
     if ld > V:
         assert torch.equal(out["dlogits"][:, V:], sentinel)   # columns >= V untouched
     assert L.leap_get_device_status() == 0              # no bounded wait gave up
@@ -67,7 +70,8 @@ def test_fused_loss_all_rows(V, ld):
     assert (~orc["active"] & orc["live"]).any()        # the clipped branch was exercised
 
 
-def test_slice_boundaries_at_vocab_151936():
+@pytest.mark.parametrize("single_read", [False, True])
+def test_slice_boundaries_at_vocab_151936(single_read):
     """Targets placed on every CTA-slice and vector boundary of the cluster split."""
     L = leap()
     V = 151936
@@ -77,7 +81,7 @@ def test_slice_boundaries_at_vocab_151936():
     z, ids, old, adv, w = _inputs(N, V, seed=11, sigma=3.0, spikes=0.01, mask_frac=0.0)
     ids.copy_(torch.tensor(targets, dtype=torch.int32))
     old.copy_(torch_logp(z, ids, V) + synth.normal(N, 0.05, 12, "cuda"))
-    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V)
+    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, single_read=single_read)
     orc = _oracle_rows(z, ids, old, adv, w, list(range(N)), V)
     _check_rows(out, orc, list(range(N)), V, dl=out["dlogits"])
 
@@ -97,6 +101,20 @@ def test_forward_only_and_split_backward_match_fused(V):
     assert abs(fused["loss"].item() - fwd["loss"].item()) <= TOL_LOSS_REL * abs(orc["loss"])
     dl = L.leap_grpo_loss_bwd(z, ids, old, adv, w, fwd["lse"], V=V)
     check_dlogits_rows(bf16_rows_to_f64(dl[:, :V]), orc, rows)
+
+
+def test_large_vocab_default_path_and_single_read_limit():
+    """The default fused kernel streams any V; the cluster kernel refuses V > 262,144."""
+    L = leap()
+    V, N = 300000, 24
+    z, ids, old, adv, w = _inputs(N, V, seed=13, sigma=3.0, spikes=0.01, old_sigma=0.3)
+    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V)
+    orc = _oracle_rows(z, ids, old, adv, w, list(range(N)), V)
+    _check_rows(out, orc, list(range(N)), V, dl=out["dlogits"])
+    assert abs(out["loss"].item() - orc["loss"]) <= TOL_LOSS_REL * abs(orc["loss"])
+    with pytest.raises(L.LeapError) as e:
+        L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, single_read=True)
+    assert e.value.status == L.LEAP_ERR_UNSUPPORTED
 
 
 @pytest.mark.parametrize("V", [1024, 1000, 151936])
