@@ -295,6 +295,48 @@ leap_status_t leap_grpo_loss_bwd(
     uint16_t* dlogits,
     void* stream);
 
+/* ------------------------------------------------------------------------
+ * 5. Fused lm-head: token log-probs straight from the hidden states, logits =
+ *    hidden . W^T computed tile by tile on the tensor cores (tcgen05) and
+ *    reduced in tensor memory, never stored; the same clipped surrogate as
+ *    section 4; and the gradient with respect to the hidden states.
+ * ------------------------------------------------------------------------ */
+
+/*
+ * Plain GEMM building block: C[M x N] = A[M x K] . B[N x K]^T with bf16
+ * inputs, fp32 accumulation on tcgen05 and bf16 output (round to nearest).
+ * A, B, C row-major with leading dimensions lda, ldb >= K and ldc >= N, all
+ * multiples of 8 elements; 16-byte aligned bases.
+ */
+leap_status_t leap_gemm_bf16_nt(const uint16_t* A, int64_t lda, const uint16_t* B, int64_t ldb,
+                                uint16_t* C, int64_t ldc, int32_t M, int32_t N, int32_t K,
+                                void* stream);
+
+/* Bytes of workspace leap_fused_lmhead_logprobs needs (with_dhidden: 0 when
+ * dhidden will be NULL).  With dhidden it includes a transposed copy of W
+ * (H x V bf16) and one 8,192-token chunk of bf16 dlogits. */
+size_t leap_fused_lmhead_workspace_size(int64_t N, int32_t H, int32_t V, int32_t with_dhidden);
+
+/*
+ * hidden bf16 [N x H] (row-major), W bf16 [V x H] (the lm-head weight,
+ * row-major); H % 8 == 0, 16-byte aligned bases.  logits z = hidden . W^T,
+ * then exactly leap_grpo_loss_fwd's outputs (loss, logp, lse, ell, stats;
+ * ids, old_logp, adv, w as there; params->flags may hold
+ * LEAP_LOSS_ACCUMULATE).  If dhidden (bf16 [N x H]) is not NULL it receives
+ * d loss / d hidden = dlogits . W, computed from bf16 dlogits of 8,192-token
+ * chunks.  workspace: >= leap_fused_lmhead_workspace_size bytes, 256-byte
+ * aligned.
+ */
+leap_status_t leap_fused_lmhead_logprobs(
+    const leap_loss_params_t* params,
+    const uint16_t* hidden, const uint16_t* W, int64_t N, int32_t H, int32_t V,
+    const int32_t* ids, const float* old_logp, const float* adv, const float* w,
+    float* loss, float* logp, float* lse, float* ell,
+    uint16_t* dhidden,
+    void* workspace, size_t ws_bytes,
+    leap_loss_stats_t* stats,
+    void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -60,6 +60,8 @@ bool rows_ok(const uint16_t* logits, int64_t ld, const int32_t* ids, int64_t N, 
 
 }  // namespace
 
+unsigned int* device_status_ptr() { return status_ptr(); }
+
 int device_sm_count() {
     const int d = current_device();
     if (d < 0) return 132;

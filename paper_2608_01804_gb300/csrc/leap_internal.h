@@ -98,5 +98,7 @@ cudaError_t launch_loss_reduce(const LossWorkspace& ws, int64_t N, float* loss, 
 int64_t fused_max_vocab();
 
 int device_sm_count();
+// Device address of the sticky status word on the current device (null on error).
+unsigned int* device_status_ptr();
 
 }  // namespace leap

@@ -42,7 +42,8 @@ EXPORTS = (
     "leap_status_string", "leap_version", "leap_get_device_status",
     "leap_group_rank_advantages", "leap_rollout_token_counts", "leap_scatter_turn_advantages",
     "leap_token_logprobs", "leap_grpo_loss_workspace_size", "leap_grpo_loss_fwd", "leap_grpo_loss_bwd",
-    "leap_grpo_loss_fwd_noalloc",
+    "leap_grpo_loss_fwd_noalloc", "leap_gemm_bf16_nt", "leap_fused_lmhead_workspace_size",
+    "leap_fused_lmhead_logprobs",
 )
 LEAP_NOALLOC_MAX_ROWS = 65536
 
@@ -108,6 +109,13 @@ def lib() -> ctypes.CDLL:
     L.leap_grpo_loss_fwd_noalloc.restype = S
     L.leap_grpo_loss_fwd_noalloc.argtypes = [ctypes.POINTER(LossParams), _P, _I64, _P, _P, _P, _P, _I64, _I32,
                                              _P, _P, _P, _P, _P, _P, _P]
+    L.leap_gemm_bf16_nt.restype = S
+    L.leap_gemm_bf16_nt.argtypes = [_P, _I64, _P, _I64, _P, _I64, _I32, _I32, _I32, _P]
+    L.leap_fused_lmhead_workspace_size.restype = _SZ
+    L.leap_fused_lmhead_workspace_size.argtypes = [_I64, _I32, _I32, _I32]
+    L.leap_fused_lmhead_logprobs.restype = S
+    L.leap_fused_lmhead_logprobs.argtypes = [ctypes.POINTER(LossParams), _P, _P, _I64, _I32, _I32, _P, _P, _P, _P,
+                                             _P, _P, _P, _P, _P, _P, _SZ, _P, _P]
     L.leap_grpo_loss_bwd.restype = S
     L.leap_grpo_loss_bwd.argtypes = [ctypes.POINTER(LossParams), _P, _I64, _P, _P, _P, _P, _P, _I64, _I32,
                                      _P, _P]
@@ -315,3 +323,61 @@ def read_stats(t) -> dict:
     s = LossStats.from_buffer_copy(raw)
     return dict(loss_sum=s.loss_sum, rho_sum=s.rho_sum, live_tokens=s.live_tokens,
                 clipped_tokens=s.clipped_tokens)
+
+
+def _bf16_2d(t, name):
+    if t.dtype != torch.bfloat16 or t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError("%s must be a 2-D bf16 tensor with contiguous rows" % name)
+    return ctypes.c_void_p(t.data_ptr()), t.stride(0)
+
+
+def leap_gemm_bf16_nt(A, B, out=None, stream=None):
+    """out[M x N] = A[M x K] . B[N x K]^T (bf16 in and out, fp32 accumulation on tcgen05)."""
+    pa, lda = _bf16_2d(A, "A")
+    pb, ldb = _bf16_2d(B, "B")
+    M, K = A.shape
+    N = B.shape[0]
+    if B.shape[1] != K:
+        raise ValueError("inner dimensions differ")
+    if out is None:   # rows padded to a multiple of 8 elements (16 bytes), returned as an [M x N] view
+        out = torch.empty((M, (N + 7) // 8 * 8), dtype=torch.bfloat16, device=A.device)[:, :N]
+    pc, ldc = _bf16_2d(out, "out")
+    st = lib().leap_gemm_bf16_nt(pa, lda, pb, ldb, pc, ldc, M, N, K, _stream(stream))
+    _check(st, "leap_gemm_bf16_nt")
+    return out
+
+
+def leap_fused_lmhead_workspace_size(N, H, V, with_dhidden=True) -> int:
+    return int(lib().leap_fused_lmhead_workspace_size(int(N), int(H), int(V), 1 if with_dhidden else 0))
+
+
+def leap_fused_lmhead_logprobs(hidden, W, ids, old_logp, adv, w, *, eps_low=0.2, eps_high=0.2, inv_temp=1.0,
+                               grad_scale=1.0, accumulate=False, want_dhidden=True, loss=None, logp=None, lse=None,
+                               ell=None, dhidden=None, workspace=None, stats=None, stream=None):
+    """Clipped-surrogate loss from hidden states and the lm-head weight (logits never stored)."""
+    ph, ldh = _bf16_2d(hidden, "hidden")
+    pw, ldw = _bf16_2d(W, "W")
+    N, H = hidden.shape
+    V = W.shape[0]
+    if ldh != H or ldw != H or W.shape[1] != H:
+        raise ValueError("hidden and W must be contiguous [N x H] and [V x H]")
+    dev = hidden.device
+    if loss is None:
+        loss = torch.zeros(1, dtype=torch.float32, device=dev)
+    logp = _empty(N, torch.float32, hidden) if logp is None else logp
+    lse = _empty(N, torch.float32, hidden) if lse is None else lse
+    ell = _empty(N, torch.float32, hidden) if ell is None else ell
+    if want_dhidden and dhidden is None:
+        dhidden = torch.empty_like(hidden)
+    if not want_dhidden:
+        dhidden = None
+    if workspace is None:
+        workspace = torch.empty(max(1, leap_fused_lmhead_workspace_size(N, H, V, want_dhidden)), dtype=torch.uint8,
+                                device=dev)
+    p = LossParams(eps_low, eps_high, inv_temp, grad_scale, LEAP_LOSS_ACCUMULATE if accumulate else 0)
+    st = lib().leap_fused_lmhead_logprobs(ctypes.byref(p), ph, pw, N, H, V, _ptr(ids), _ptr(old_logp), _ptr(adv),
+                                          _ptr(w), _ptr(loss), _ptr(logp), _ptr(lse), _ptr(ell),
+                                          None if dhidden is None else ctypes.c_void_p(dhidden.data_ptr()),
+                                          _ptr(workspace), workspace.numel(), _ptr(stats), _stream(stream))
+    _check(st, "leap_fused_lmhead_logprobs")
+    return dict(loss=loss, logp=logp, lse=lse, ell=ell, dhidden=dhidden)

@@ -1,0 +1,92 @@
+"""GPU parity of the tcgen05 path: the plain GEMM against torch's fp32 matmul of
+the same bf16 values, and the fused lm-head (log-probs, loss, dhidden)
+against the fp64 oracle.
+
+Tolerances: the GEMM output is bf16 of an fp32 sum, so |C - ref| <= one bf16
+ulp of |ref| plus fp32 accumulation slack (1e-4 of the row's largest
+|ref|).  dhidden is a sum over V of bf16-rounded dlogits (relative 2^-9 each)
+rounded once more to bf16, so its normwise relative error per row is bounded
+by about 2^-8: the test uses 1e-2.  Log-probs 2e-3 absolute, loss 1e-4
+relative, as everywhere."""
+import numpy as np
+import pytest
+import torch
+
+from harness import O, TOL_LOGP, TOL_LOSS_REL, bf16_rows_to_f64, leap
+
+pytestmark = pytest.mark.gpu
+
+
+def _bf16(shape, sigma, seed):
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    return (torch.randn(shape, generator=g, device="cuda") * sigma).to(torch.bfloat16)
+
+
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (256, 512, 320), (200, 300, 136), (1000, 1000, 1024),
+                                   (130, 520, 5120)])
+def test_gemm_bf16_nt(M, N, K):
+    L = leap()
+    A = _bf16((M, K), 1.0, M + K)
+    B = _bf16((N, K), 0.5, N + 3 * K)
+    C = L.leap_gemm_bf16_nt(A, B)
+    ref = (A.double() @ B.double().T)
+    got = C.double()
+    bound = 2.0 ** -8 * ref.abs() + 1e-4 * ref.abs().amax(dim=1, keepdim=True) + 1e-30
+    bad = (got - ref).abs() > bound
+    assert not bad.any(), "max excess %r at %r" % (((got - ref).abs() - bound).max().item(),
+                                                   torch.nonzero(bad)[:5].tolist())
+
+
+def _lmhead_inputs(N, H, V, seed, old_sigma=0.3):
+    hidden = _bf16((N, H), 1.0, seed)
+    W = _bf16((V, H), 0.02 * 8, seed + 1)     # wider logits than 0.02 so the softmax is not flat
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed + 2)
+    ids = torch.randint(0, V, (N,), generator=g, device="cuda", dtype=torch.int32)
+    z = hidden.float() @ W.float().T
+    logp = torch.log_softmax(z, dim=1).gather(1, ids.long().view(-1, 1)).view(-1)
+    old = logp + torch.randn(N, generator=g, device="cuda") * old_sigma
+    rng = np.random.default_rng(seed)
+    adv = torch.as_tensor(rng.normal(0, 1, N).astype(np.float32), device="cuda")
+    w = rng.uniform(0.01, 0.1, N).astype(np.float32)
+    w[rng.random(N) < 0.25] = 0.0
+    return hidden, W, ids, old, adv, torch.as_tensor(w, device="cuda")
+
+
+@pytest.mark.parametrize("N,H,V", [(128, 64, 256), (300, 256, 1000), (520, 512, 4100), (256, 1024, 32000)])
+def test_fused_lmhead_all_rows(N, H, V):
+    L = leap()
+    L.leap_get_device_status()
+    hidden, W, ids, old, adv, w = _lmhead_inputs(N, H, V, seed=N + V)
+    out = L.leap_fused_lmhead_logprobs(hidden, W, ids, old, adv, w)
+    torch.cuda.synchronize()
+    assert L.leap_get_device_status() == 0
+    hf = bf16_rows_to_f64(hidden)
+    Wf = bf16_rows_to_f64(W)
+    orc = O.lmhead_loss_rows(hf, Wf, ids.cpu().numpy(), old.cpu().numpy().astype(np.float64),
+                             adv.cpu().numpy().astype(np.float64), w.cpu().numpy().astype(np.float64))
+    live = orc["live"]
+    logp = out["logp"].cpu().numpy().astype(np.float64)
+    assert np.max(np.abs(logp - orc["logp"])) <= TOL_LOGP
+    assert np.all(logp[~live] == 0)
+    np.testing.assert_allclose(out["lse"].cpu().numpy()[live], orc["lse"][live], rtol=1e-5)
+    assert abs(out["loss"].item() - orc["loss"]) <= TOL_LOSS_REL * abs(orc["loss"])
+    dh = bf16_rows_to_f64(out["dhidden"])
+    ref = orc["dhidden"]
+    for k in range(N):
+        nrm = np.linalg.norm(ref[k])
+        if nrm == 0:
+            assert np.all(dh[k] == 0)
+        else:
+            assert np.linalg.norm(dh[k] - ref[k]) <= 1e-2 * nrm, (k, np.linalg.norm(dh[k] - ref[k]) / nrm)
+
+
+def test_fused_lmhead_forward_only():
+    L = leap()
+    hidden, W, ids, old, adv, w = _lmhead_inputs(256, 128, 3000, seed=5)
+    out = L.leap_fused_lmhead_logprobs(hidden, W, ids, old, adv, w, want_dhidden=False)
+    assert out["dhidden"] is None
+    full = L.leap_fused_lmhead_logprobs(hidden, W, ids, old, adv, w)
+    assert out["loss"].item() == full["loss"].item()
+    assert torch.equal(out["logp"], full["logp"])
