@@ -62,6 +62,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-rows", action="store_true", help="skip the per-row measurements")
+    ap.add_argument("--lmhead-tokens", type=int, default=0,
+                    help="run only the fused lm-head (forward + dhidden) on this many tokens, for profiling captures")
     ap.add_argument("--prompts", type=int, default=16,
                     help="prompts per rank (16 = the benchmark workload; fewer only for profiling captures)")
     return ap.parse_args()
@@ -72,6 +74,14 @@ def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return rank, world, local
+
+
+def measured_tensor_peak():
+    """Sustained dense bf16 TFLOP/s (the lm-head kernels run for tens of ms)."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        return float(json.load(open(p))["bf16_tflops_sustained"])
+    return 1700.0
 
 
 def measured_peaks():
@@ -322,15 +332,81 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
     split = entry(6 * V * live + 2 * V * (N - live) + 36 * N, ms_f + ms_b, live, "valid tokens/s")
     split["frac_vs_fused_4V_bytes"] = (4 * V * live + 2 * V * (N - live) + 16 * N) / ((ms_f + ms_b) / 1e3) / 1e9 / peak
     rows["split_fwd_then_bwd_32768xV"] = split
-    del dl, ws, flush_buf
+    del dl, ws
+    torch.cuda.synchronize()
+
+    # a8: fused lm-head (tcgen05), 65,536 tokens x H = 5,120 x V = 151,936.
+    from paper_2608_01804_gb300.step import GrpoStep
+    lb = synth.lmhead_batch()
+    N8, H = lb.N, 5120
+    hidden = synth.normal((N8, H), 1.0, 500, device, dtype=torch.bfloat16)
+    W = synth.normal((V, H), 0.02, 501, device, dtype=torch.bfloat16)
+    ids8 = synth.token_ids(N8, V, 502, device)
+    old8 = torch.empty(N8, dtype=torch.float32, device=device)
+    for a0 in range(0, N8, 4096):     # current-policy log-probs (torch), input generation only
+        zc = (hidden[a0:a0 + 4096] @ W.T).float()
+        old8[a0:a0 + 4096] = torch.log_softmax(zc, 1).gather(1, ids8[a0:a0 + 4096].long().view(-1, 1)).view(-1)
+        del zc
+    old8 += synth.normal(N8, 0.05, 503, device)
+    st8 = GrpoStep(lb, V, device, gamma=1.0, tau=(0, lb.G), use_gate_in=False)
+    st8.advantages()
+    ws8 = torch.empty(L.leap_fused_lmhead_workspace_size(N8, H, V, True), dtype=torch.uint8, device=device)
+    dh = torch.empty_like(hidden)
+    fwd8 = lambda: L.leap_fused_lmhead_logprobs(hidden, W, ids8, old8, st8.adv, st8.w, want_dhidden=False,
+                                                workspace=ws8)
+    full8 = lambda: L.leap_fused_lmhead_logprobs(hidden, W, ids8, old8, st8.adv, st8.w, dhidden=dh, workspace=ws8)
+    fwd8()
+    full8()
+    tpeak = measured_tensor_peak()
+    ms = _timed_launches(fwd8, 3, stream)
+    fl = 2.0 * N8 * V * H
+    rows["fused_lmhead_fwd_65536x5120xV"] = {"ms": ms, "algorithmic_flops": fl, "achieved_tflops": fl / ms / 1e9,
+                                            "frac": fl / ms / 1e9 / tpeak, "throughput": N8 / (ms / 1e3),
+                                            "unit": "tokens/s", "bound": "tensor"}
+    ms = _timed_launches(full8, 3, stream)
+    fl = 6.0 * N8 * V * H
+    rows["fused_lmhead_fwd_dhidden_65536x5120xV"] = {"ms": ms, "algorithmic_flops": fl,
+                                                     "achieved_tflops": fl / ms / 1e9,
+                                                     "frac": fl / ms / 1e9 / tpeak, "throughput": N8 / (ms / 1e3),
+                                                     "unit": "tokens/s", "bound": "tensor"}
+    del hidden, W, dh, ws8, flush_buf
     torch.cuda.synchronize()
     return rows
+
+
+def lmhead_only(args):
+    """The fused lm-head alone (H = 5,120, V = 151,936) on --lmhead-tokens tokens:
+    --warmup untimed calls, then --steps timed ones; prints one JSON line."""
+    from paper_2608_01804_gb300 import build
+    build.build()
+    from paper_2608_01804_gb300 import leap as L
+    from paper_2608_01804_gb300 import synth
+    device = torch.device("cuda", 0)
+    N, H = args.lmhead_tokens, 5120
+    hidden = synth.normal((N, H), 1.0, 500, device, dtype=torch.bfloat16)
+    W = synth.normal((V, H), 0.02, 501, device, dtype=torch.bfloat16)
+    ids = synth.token_ids(N, V, 502, device)
+    old = synth.normal(N, 1.0, 503, device) - 12.0
+    adv = synth.normal(N, 1.0, 504, device)
+    w = torch.full((N,), 1.0 / N, device=device)
+    ws = torch.empty(L.leap_fused_lmhead_workspace_size(N, H, V, True), dtype=torch.uint8, device=device)
+    dh = torch.empty_like(hidden)
+    run = lambda: L.leap_fused_lmhead_logprobs(hidden, W, ids, old, adv, w, dhidden=dh, workspace=ws)
+    for _ in range(args.warmup):
+        run()
+    ms = _timed_launches(run, args.steps, torch.cuda.current_stream())
+    fl = 6.0 * N * V * H
+    print(json.dumps({"lmhead_tokens": N, "ms": ms, "tflops": fl / ms / 1e9,
+                      "frac": fl / ms / 1e9 / measured_tensor_peak()}), flush=True)
 
 
 def main():
     args = parse_args()
     if args.impl == "reference":
         reference_arm(args)
+        return
+    if args.lmhead_tokens:
+        lmhead_only(args)
         return
     rank, world, local = dist_env()
     torch.cuda.set_device(local)

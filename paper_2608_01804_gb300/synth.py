@@ -189,6 +189,13 @@ def shard(batch, rank, world):
                         batch.seg_turn[s0:s1].copy(), info=info)
 
 
+def lmhead_batch(seed=4, n_rollouts=8, tokens=8192):
+    """One group of `n_rollouts` single-turn rollouts of `tokens` response tokens
+    each, every token valid (the fused lm-head workload: 8 x 8,192 = 65,536
+    tokens), pass ~ Bernoulli(0.5)."""
+    return padded_batch(1, n_rollouts, 1, tokens, 0.5, tokens, tokens, seed, gate_in=None)
+
+
 def tournament_outcomes(seed=3, num_groups=65536, G=64, M=3, dup_frac=0.1):
     """Outcome tuples only (no tokens): pass ~ Bernoulli(0.5), turn index ~ U{1..M},
     speedup ~ LogNormal(0, 1), tokens ~ U{128..8192}; about `dup_frac` of the

@@ -90,3 +90,43 @@ def test_fused_lmhead_forward_only():
     full = L.leap_fused_lmhead_logprobs(hidden, W, ids, old, adv, w)
     assert out["loss"].item() == full["loss"].item()
     assert torch.equal(out["logp"], full["logp"])
+
+
+def test_fused_lmhead_full_size_sampled():
+    """65,536 tokens x H = 5,120 x V = 151,936 (the benchmark's lm-head workload):
+    sampled rows against the oracle; the loss against the fp64 sum of the
+    kernel's own per-row terms."""
+    from paper_2608_01804_gb300 import synth
+    L = leap()
+    N, H, V = 65536, 5120, 151936
+    hidden = synth.normal((N, H), 1.0, 600, "cuda", dtype=torch.bfloat16)
+    W = synth.normal((V, H), 0.02, 601, "cuda", dtype=torch.bfloat16)
+    ids = synth.token_ids(N, V, 602, "cuda")
+    rng = np.random.default_rng(603)
+    rows = sorted(set([0, 1, 127, 128, N - 1] + rng.choice(N, 7, replace=False).tolist()))
+    sel = torch.as_tensor(rows, device="cuda")
+    z_sel = (hidden[sel].float() @ W.float().T)
+    old = torch.full((N,), -12.0, device="cuda")
+    old[sel] = torch.log_softmax(z_sel, 1).gather(1, ids[sel].long().view(-1, 1)).view(-1) + 0.3
+    adv = torch.as_tensor(rng.normal(0, 1, N).astype(np.float32), device="cuda")
+    w = torch.full((N,), 1.0 / N, device="cuda")
+    w[rows[2]] = 0.0
+    out = L.leap_fused_lmhead_logprobs(hidden, W, ids, old, adv, w)
+    torch.cuda.synchronize()
+    assert L.leap_get_device_status() == 0
+    Wf = bf16_rows_to_f64(W)
+    hf = bf16_rows_to_f64(hidden[sel])
+    orc = O.lmhead_loss_rows(hf, Wf, ids[sel].cpu().numpy(), old[sel].cpu().numpy().astype(np.float64),
+                             adv[sel].cpu().numpy().astype(np.float64), w[sel].cpu().numpy().astype(np.float64))
+    logp = out["logp"][sel].cpu().numpy().astype(np.float64)
+    assert np.max(np.abs(logp - orc["logp"])) <= TOL_LOGP
+    np.testing.assert_allclose(out["ell"][sel].cpu().numpy(), orc["ell"], rtol=1e-4, atol=1e-7)
+    dh = bf16_rows_to_f64(out["dhidden"][sel])
+    for k in range(len(rows)):
+        nrm = np.linalg.norm(orc["dhidden"][k])
+        if nrm == 0:
+            assert np.all(dh[k] == 0)
+        else:
+            assert np.linalg.norm(dh[k] - orc["dhidden"][k]) <= 1e-2 * nrm
+    tot = float((w.double() * out["ell"].double()).sum().item())
+    assert abs(out["loss"].item() - tot) <= 1e-6 * abs(tot) + 1e-12
