@@ -41,7 +41,8 @@ WORKLOAD = ("single-turn GRPO: 16 prompts x G=8 x 256 token slots = 32,768 rows 
 # kernel built from sources with this SHA-256 on a 4,096-row slice, scaled to the full launch by
 # algorithmic bytes (traffic grows in proportion to them); null once the sources change.
 KNOWN_TRAFFIC = {"src_sha256": "719d7f95fc58e9df03814195268dd11a1da3831c83618cee9e3bb9d4593f1fb1", "bytes_per_launch": 16099568938}
-KERNEL_SOURCES = ("paper_2608_01804_gb300/csrc/logprob_loss.cu", "paper_2608_01804_gb300/csrc/leap_common.cuh")
+KERNEL_SOURCES = ("paper_2608_01804_gb300/csrc/logprob_loss.cu", "paper_2608_01804_gb300/csrc/leap_common.cuh",
+                  "paper_2608_01804_gb300/csrc/loss_math.cuh")
 
 
 def _src_sha():

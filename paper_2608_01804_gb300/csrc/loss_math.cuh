@@ -26,6 +26,11 @@ __device__ __forceinline__ TokenLoss token_loss(const RowArgs& a, float m, float
     r.ell = -fminf(r.rho * A, clipped * A);
     r.active = (A >= 0.f) ? (r.rho <= hi) : (r.rho >= lo);
     r.g = r.active ? -wk * A * r.rho : 0.f;
+    if (isnan(r.rho)) {  // fminf / fmaxf would drop a NaN: keep it in the loss and the gradient
+        r.ell = r.rho;
+        r.g = r.rho;
+        r.active = false;
+    }
     return r;
 }
 
