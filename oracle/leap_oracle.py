@@ -33,6 +33,10 @@ AGG_SEQ_MEAN_TOKEN_MEAN = 0
 AGG_TOKEN_MEAN = 1
 ADVNORM_GRPO_STD = 0
 ADVNORM_NONE = 1
+CMP_PAPER = 0
+CMP_LEXI = 1
+REWARD_RANK = 0
+REWARD_STATIC = 1
 
 
 # ---------------------------------------------------------------------------
@@ -92,6 +96,44 @@ def tournament(r):
     return n_worse, n_better
 
 
+def tournament_lexi(r, speedup, ntokens):
+    """Extension of Eq. 5 with tie-breaks (not in the paper): rollout i beats j
+    if its tier is higher, or the tiers are equal, both passed (r > 0), and i
+    has the higher speedup, or the same speedup and fewer tokens.  Failures
+    (r = 0) carry no speedup and tie among themselves; exact ties count in
+    neither direction.  Pairwise double loop, vectorised over groups."""
+    r = np.asarray(r, dtype=np.int64)
+    sp = np.asarray(speedup, dtype=np.float64)
+    tk = np.asarray(ntokens, dtype=np.int64)
+    num_groups, G = r.shape
+    n_worse = np.zeros((num_groups, G), dtype=np.int64)
+    n_better = np.zeros((num_groups, G), dtype=np.int64)
+
+    def beats(a, b):
+        ra, rb = r[:, a:a + 1], r[:, b]
+        sa, sb = sp[:, a:a + 1], sp[:, b]
+        ta, tb = tk[:, a:a + 1], tk[:, b]
+        return (ra > rb) | ((ra == rb) & (ra > 0) & ((sa > sb) | ((sa == sb) & (ta < tb))))
+
+    allj = np.arange(G)
+    for i in range(G):
+        others = allj != i
+        n_worse[:, i] = np.sum(beats(i, allj) & others, axis=1)
+        # j beats i, for every j: evaluate with j as the first argument
+        better = (r > r[:, i:i + 1]) | ((r == r[:, i:i + 1]) & (r > 0) &
+                                        ((sp > sp[:, i:i + 1]) | ((sp == sp[:, i:i + 1]) & (tk < tk[:, i:i + 1]))))
+        n_better[:, i] = np.sum(better & others, axis=1)
+    return n_worse, n_better
+
+
+def static_reward(r, M, c):
+    """The static-scalar multi-turn reward the paper compares against (Sec. 3.2,
+    "GRPO-MT" in Table 6): 1 for a first-turn pass, the constant c for a pass
+    at a later turn, 0 for a failure."""
+    r = np.asarray(r, dtype=np.int64)
+    return np.where(r == M, 1.0, np.where(r > 0, float(c), 0.0))
+
+
 def tournament_reward(n_worse, n_better, G):
     """Eq. 6: R_i = (N_worse(o_i) - N_better(o_i)) / (G - 1), in [-1, 1]."""
     if G < 2:
@@ -139,18 +181,50 @@ def turn_advantages(A, T_eff, gamma, M):
 
 def rank_advantages(pass_turn, num_turns, M, tau_min, tau_max, gamma,
                     eps_std=1e-6, norm=ADVNORM_GRPO_STD, std_unbiased=True,
-                    gate_in=None):
-    """Sec. 3.1-3.3 end to end for every group: gate, tiers, tournament, R, A, A_hat."""
+                    gate_in=None, cmp=CMP_PAPER, speedup=None, ntokens=None,
+                    reward=REWARD_RANK, static_c=0.5):
+    """Sec. 3.1-3.3 end to end for every group: gate, tiers, tournament, R, A, A_hat.
+
+    reward = REWARD_STATIC replaces the tournament reward by the static-scalar
+    baseline (tiers and counts are still reported)."""
     pass_turn = np.asarray(pass_turn)
     G = pass_turn.shape[1]
     n_fail, gate, r, T_eff, bad = tiers_and_gate(pass_turn, num_turns, M,
                                                  tau_min, tau_max, gate_in)
-    n_worse, n_better = tournament(r)
-    R = tournament_reward(n_worse, n_better, G)
+    if cmp == CMP_LEXI:
+        n_worse, n_better = tournament_lexi(r, np.asarray(speedup).reshape(r.shape),
+                                            np.asarray(ntokens).reshape(r.shape))
+    else:
+        n_worse, n_better = tournament(r)
+    if reward == REWARD_STATIC:
+        R = static_reward(r, M, static_c)
+    else:
+        R = tournament_reward(n_worse, n_better, G)
     A = grpo_advantage(R, eps_std, norm, std_unbiased)
     turn_adv = turn_advantages(A, T_eff, gamma, M)
     return dict(n_fail=n_fail, gate=gate, r=r, T_eff=T_eff, bad_outcome=bad,
                 n_worse=n_worse, n_better=n_better, R=R, A=A, turn_adv=turn_adv)
+
+
+def rank_stats(out, pass_turn, M):
+    """Training-observability counters (Table 5, Sec. 4.2) from rank_advantages'
+    results: activated groups, per-rollout and per-group recovery, passes by
+    turn, total effective turns and passed samples (turns per pass)."""
+    gate = np.asarray(out["gate"]).astype(bool)
+    T_eff = np.asarray(out["T_eff"])
+    bad = np.asarray(out["bad_outcome"])
+    pt = np.where(bad, 0, np.asarray(pass_turn, dtype=np.int64))
+    on = gate[:, None] & ~bad
+    first = (pt == 1) & ~bad
+    later = on & (pt >= 2)                              # recovered after a first-turn failure
+    failed_first_on = on & (pt != 1)
+    passes_by_turn = [int(np.sum(first)) if m == 1 else int(np.sum(later & (pt == m))) for m in range(1, 9)]
+    return dict(groups=int(gate.size), gated_groups=int(gate.sum()), rollouts=int(pt.size),
+                nonzero_adv_rollouts=int(np.count_nonzero(np.abs(out["A"]) > 1e-9)),
+                first_turn_passes=int(first.sum()), later_passes=int(later.sum()),
+                groups_with_recovery=int(np.sum(np.any(later, axis=1))),
+                failed_first_turn_in_gated=int(failed_first_on.sum()),
+                total_turns=int(T_eff.sum()), passes_by_turn=passes_by_turn)
 
 
 # ---------------------------------------------------------------------------

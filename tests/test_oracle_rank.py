@@ -230,3 +230,66 @@ def test_turn_discount_properties():
                     else:
                         assert ta[g, i, t] == A[g, i]
                 assert np.all(ta[g, i, T[g, i]:] == 0)
+
+
+# ---- extensions: lexicographic tie-breaks, static-scalar baseline, counters ----
+
+def _lexi_brute(r, sp, tk):
+    """Python tuple ordering as an independent formulation of the tie-broken
+    tournament: passing rollouts carry (r, speedup, -tokens), failures (0,)."""
+    keys = [(int(a), float(b), -int(c)) if a > 0 else (0,) for a, b, c in zip(r, sp, tk)]
+    nw = [sum(1 for j, kj in enumerate(keys) if j != i and ki > kj) for i, ki in enumerate(keys)]
+    nb = [sum(1 for j, kj in enumerate(keys) if j != i and ki < kj) for i, ki in enumerate(keys)]
+    return np.array(nw), np.array(nb)
+
+
+def test_lexi_tournament_against_tuple_ordering():
+    rng = np.random.default_rng(21)
+    for G in (2, 5, 8, 33):
+        r = rng.integers(0, 4, size=(6, G))
+        sp = rng.choice([0.5, 1.0, 1.5], size=(6, G))          # many exact ties
+        tk = rng.choice([100, 200], size=(6, G))
+        nw, nb = O.tournament_lexi(r, sp, tk)
+        for g in range(6):
+            bw, bb = _lexi_brute(r[g], sp[g], tk[g])
+            np.testing.assert_array_equal(nw[g], bw)
+            np.testing.assert_array_equal(nb[g], bb)
+        np.testing.assert_array_equal(nw.sum(axis=1), nb.sum(axis=1))
+
+
+def test_lexi_reduces_to_paper_comparator_without_tie_breaks():
+    rng = np.random.default_rng(22)
+    r = rng.integers(0, 4, size=(10, 16))
+    nw, nb = O.tournament_lexi(r, np.ones_like(r, dtype=float), np.full(r.shape, 7))
+    pw, pb = O.tournament(r)
+    np.testing.assert_array_equal(nw, pw)
+    np.testing.assert_array_equal(nb, pb)
+
+
+def test_static_reward_baseline_by_hand():
+    """GRPO-MT baseline, G = 4, M = 2, c = 0.5: outcomes (turn-1 pass, turn-2
+    pass, fail, fail) -> R = (1, 0.5, 0, 0), mean 0.375, unbiased std
+    sqrt(0.6875 / 3); A worked out by hand."""
+    out = _run([1, 2, 0, 0], 2, reward=O.REWARD_STATIC, static_c=0.5, eps_std=0.0)
+    np.testing.assert_allclose(out["R"][0], [1.0, 0.5, 0.0, 0.0])
+    std = np.sqrt(0.6875 / 3)
+    np.testing.assert_allclose(out["A"][0], np.array([0.625, 0.125, -0.375, -0.375]) / std, rtol=1e-12)
+    # Single turn: the static reward is the binary reward, so A equals the rank-based A.
+    a = _run([1, 0, 1, 1, 0], 1, reward=O.REWARD_STATIC, eps_std=0.0)["A"]
+    b = _run([1, 0, 1, 1, 0], 1, eps_std=0.0)["A"]
+    np.testing.assert_allclose(a, b, rtol=1e-12)
+
+
+def test_rank_stats_by_hand():
+    """Two groups of 4, M = 3.  Group 0 gated on: turn-1 pass, turn-2 pass,
+    turn-3 pass, fail (T = 1, 2, 3, 3).  Group 1 gated off: pass, fail, fail,
+    turn-2 pass truncated to a failure."""
+    pt = np.array([[1, 2, 3, 0], [1, 0, 0, 2]])
+    nt = np.array([[1, 2, 3, 3], [1, 1, 1, 2]])
+    out = O.rank_advantages(pt, nt, 3, 0, 4, 0.9, gate_in=np.array([1, 0]))
+    st = O.rank_stats(out, pt, 3)
+    assert (st["groups"], st["gated_groups"], st["rollouts"]) == (2, 1, 8)
+    assert (st["first_turn_passes"], st["later_passes"]) == (2, 2)
+    assert (st["groups_with_recovery"], st["failed_first_turn_in_gated"]) == (1, 3)
+    assert st["total_turns"] == 1 + 2 + 3 + 3 + 4
+    assert st["passes_by_turn"][:3] == [2, 1, 1]
