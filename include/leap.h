@@ -86,6 +86,30 @@ typedef enum {
     LEAP_ADVNORM_NONE = 1       /* A = R */
 } leap_advnorm_t;
 
+typedef enum {
+    LEAP_REWARD_RANK = 0,    /* Eq. 6: tournament reward (the method) */
+    LEAP_REWARD_STATIC = 1   /* static-scalar baseline the paper compares against (Sec. 3.2,
+                                Table 6 "GRPO-MT"): 1 for a turn-1 pass, static_c for a later
+                                pass, 0 for a failure */
+} leap_reward_t;
+
+/* Training-observability counters of a leap_group_rank_advantages call
+ * (Table 5, Sec. 4.2).  Device struct, ACCUMULATED (+=): zero it first.
+ *   activated-group rate  = gated_groups / groups
+ *   per-rollout recovery  = later_passes / failed_first_turn_in_gated
+ *   per-group recovery    = groups_with_recovery / gated_groups
+ *   turns per pass        = total_turns / (first_turn_passes + later_passes) */
+typedef struct {
+    int64_t groups, gated_groups;
+    int64_t rollouts, nonzero_adv_rollouts;
+    int64_t first_turn_passes;          /* passes at turn 1 (any group) */
+    int64_t later_passes;               /* passes at turn > 1 in gated groups (recoveries) */
+    int64_t groups_with_recovery;       /* gated groups with at least one recovery */
+    int64_t failed_first_turn_in_gated; /* rollouts of gated groups that failed turn 1 */
+    int64_t total_turns;                /* sum of the effective turn counts */
+    int64_t passes_by_turn[8];          /* [m - 1]: passes at turn m (turn 1 from any group) */
+} leap_rank_stats_t;
+
 typedef struct {
     int32_t num_groups;   /* prompts q in this call, >= 0 */
     int32_t G;            /* rollouts per group, 2 .. 1024 (Eq. 6 divides by G - 1) */
@@ -97,6 +121,8 @@ typedef struct {
     int32_t cmp;          /* leap_cmp_t */
     int32_t norm;         /* leap_advnorm_t */
     int32_t std_unbiased; /* 1: std divides by G - 1; 0: by G */
+    int32_t reward;       /* leap_reward_t */
+    float static_c;       /* in [0, 1]: LEAP_REWARD_STATIC's later-pass reward */
 } leap_rank_params_t;
 
 /*
@@ -111,10 +137,15 @@ typedef struct {
  *   A_i     = R_i / (std_g R + eps_std)  (mean_g R is exactly 0)     (GRPO step)
  *   turn_adv[i*M + t] = beta_i^(T_eff_i - t - 1) * A_i for t < T_eff_i, else 0,
  *             beta_i = gamma if A_i >= 0 else 1                     (Sec. 3.3)
+ * With LEAP_CMP_LEXI (an extension, not in the paper) a tie of tiers between
+ * two passing rollouts is broken by the higher speedup, then by fewer tokens;
+ * failures tie among themselves.  With LEAP_REWARD_STATIC, R is the static
+ * baseline reward and A its standard GRPO advantage (general mean; a group
+ * with all rewards equal gets A = 0).
  * Inputs  pass_turn int8 [n]: 0 = never passed, 1..M = turn of the first pass;
  *         num_turns int8 [n]: generated turns T_i, 1..M, >= pass_turn if passed;
- *         speedup f32 [n], ntokens int32 [n]: only read for LEAP_CMP_LEXI (may be NULL);
- *         gate_in u8 [num_groups] or NULL.
+ *         speedup f32 [n], ntokens int32 [n]: required for LEAP_CMP_LEXI, else ignored;
+ *         gate_in u8 [num_groups] or NULL; stats: leap_rank_stats_t or NULL.
  * Outputs (n = num_groups*G): gate_out u8 [num_groups], r_out u8 [n],
  *         n_worse, n_better int32 [n], R, A f32 [n] - each may be NULL;
  *         turn_adv f32 [n*M] and T_eff u8 [n] are required.
@@ -128,6 +159,7 @@ leap_status_t leap_group_rank_advantages(
     const uint8_t* gate_in,
     uint8_t* gate_out, uint8_t* r_out, int32_t* n_worse, int32_t* n_better,
     float* R, float* A, float* turn_adv, uint8_t* T_eff,
+    leap_rank_stats_t* stats,
     void* stream);
 
 /* ------------------------------------------------------------------------

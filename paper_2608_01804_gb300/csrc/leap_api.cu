@@ -112,7 +112,8 @@ leap_status_t leap_group_rank_advantages(const leap_rank_params_t* p, const int8
                                          const int8_t* num_turns, const float* speedup, const int32_t* ntokens,
                                          const uint8_t* gate_in, uint8_t* gate_out, uint8_t* r_out,
                                          int32_t* n_worse, int32_t* n_better, float* R, float* A,
-                                         float* turn_adv, uint8_t* T_eff, void* stream) {
+                                         float* turn_adv, uint8_t* T_eff, leap_rank_stats_t* stats,
+                                         void* stream) {
     if (!p) return LEAP_ERR_INVALID_ARG;
     if (p->num_groups < 0 || p->G < 2 || p->G > 1024 || p->M < 1 || p->M > 8) return LEAP_ERR_INVALID_ARG;
     if (!gate_in && (p->tau_min < 0 || p->tau_min > p->tau_max || p->tau_max > p->G)) return LEAP_ERR_INVALID_ARG;
@@ -121,10 +122,10 @@ leap_status_t leap_group_rank_advantages(const leap_rank_params_t* p, const int8
     if (p->norm != LEAP_ADVNORM_GRPO_STD && p->norm != LEAP_ADVNORM_NONE) return LEAP_ERR_INVALID_ARG;
     if (p->std_unbiased != 0 && p->std_unbiased != 1) return LEAP_ERR_INVALID_ARG;
     if (p->cmp != LEAP_CMP_PAPER && p->cmp != LEAP_CMP_LEXI) return LEAP_ERR_INVALID_ARG;
-    if (p->cmp == LEAP_CMP_LEXI) return LEAP_ERR_UNSUPPORTED;
+    if (p->reward != LEAP_REWARD_RANK && p->reward != LEAP_REWARD_STATIC) return LEAP_ERR_INVALID_ARG;
+    if (!finite(p->static_c) || p->static_c < 0.f || p->static_c > 1.f) return LEAP_ERR_INVALID_ARG;
     if (p->num_groups > 0 && (!pass_turn || !num_turns || !turn_adv || !T_eff)) return LEAP_ERR_INVALID_ARG;
-    (void)speedup;
-    (void)ntokens;
+    if (p->num_groups > 0 && p->cmp == LEAP_CMP_LEXI && (!speedup || !ntokens)) return LEAP_ERR_INVALID_ARG;
     RankArgs a;
     a.num_groups = p->num_groups;
     a.G = p->G;
@@ -136,6 +137,9 @@ leap_status_t leap_group_rank_advantages(const leap_rank_params_t* p, const int8
     a.cmp = p->cmp;
     a.norm = p->norm;
     a.std_unbiased = p->std_unbiased;
+    a.reward = p->reward;
+    a.static_c = p->static_c;
+    a.stats = stats;
     a.pass_turn = pass_turn;
     a.num_turns = num_turns;
     a.speedup = speedup;

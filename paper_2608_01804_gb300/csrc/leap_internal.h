@@ -10,7 +10,8 @@ namespace leap {
 struct RankArgs {
     int32_t num_groups, G, M, tau_min, tau_max;
     float gamma, eps_std;
-    int32_t cmp, norm, std_unbiased;
+    int32_t cmp, norm, std_unbiased, reward;
+    float static_c;
     const int8_t* pass_turn;
     const int8_t* num_turns;
     const float* speedup;
@@ -24,6 +25,7 @@ struct RankArgs {
     float* A;
     float* turn_adv;
     uint8_t* T_eff;
+    void* stats;  // leap_rank_stats_t*, accumulated
     unsigned int* status;
 };
 

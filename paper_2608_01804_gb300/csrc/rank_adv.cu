@@ -9,6 +9,7 @@
 #include "leap_common.cuh"
 #include "leap_internal.h"
 
+#include <algorithm>
 #include <math.h>
 
 namespace leap {
@@ -16,129 +17,264 @@ namespace {
 
 constexpr int kMaxM = 8;
 
-template <int J>  // rollouts per lane: G <= 32 * J
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Per-warp running counters (lane 0), reduced per block then added atomically.
+constexpr int kNumStats = 9 + kMaxM;
+
+template <int J, bool LEXI>  // rollouts per lane: G <= 32 * J; tie-broken comparator
 __global__ void __launch_bounds__(256) rank_adv_kernel(RankArgs a) {
     const int lane = threadIdx.x & 31;
-    const int64_t group = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (group >= a.num_groups) return;
+    const int wib = threadIdx.x >> 5;
     const int G = a.G, M = a.M;
-    const int64_t base = group * G;
-
-    int r[J], T[J];
-    bool valid[J], bad[J];
-    int n_fail = 0;
-#pragma unroll
-    for (int j = 0; j < J; ++j) {
-        const int i = lane + 32 * j;
-        valid[j] = i < G;
-        int pt = 0, nt = 1;
-        if (valid[j]) {
-            pt = a.pass_turn[base + i];
-            nt = a.num_turns[base + i];
-        }
-        bad[j] = valid[j] && (pt < 0 || pt > M || nt < 1 || nt > M || (pt >= 1 && pt > nt));
-        // Eq. 1 over first-turn outcomes; a malformed outcome counts as failed.
-        const bool fail1 = valid[j] && (bad[j] || pt != 1);
-        n_fail += __popc(__ballot_sync(0xffffffffu, fail1));
-        r[j] = pt;   // temporarily the pass turn
-        T[j] = nt;
-    }
-    // Eq. 2 (or the recorded gate).
-    const bool gate = a.gate_in ? (a.gate_in[group] != 0) : (a.tau_min <= n_fail && n_fail <= a.tau_max);
-
-    // Tier rule of Sec. 3.2; gated-off groups ran turn 1 only.
-#pragma unroll
-    for (int j = 0; j < J; ++j) {
-        const int pt = r[j];
-        if (!valid[j] || bad[j]) {
-            r[j] = 0;
-            T[j] = 0;
-        } else if (!gate) {
-            r[j] = (pt == 1) ? M : 0;
-            T[j] = 1;
-        } else {
-            r[j] = (pt >= 1) ? (M - pt + 1) : 0;
-        }
-        if (bad[j]) flag_status(a.status, 2u);
+    constexpr bool lexi = LEXI;
+    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    __shared__ long long sst[8][kNumStats];  // per-warp counters (only with a.stats)
+    if (a.stats) {
+        for (int k = lane; k < kNumStats; k += 32) sst[wib][k] = 0;
+        __syncwarp();
     }
 
-    // Histogram of tiers 0..M via ballots.
-    int hist[kMaxM + 1];
+    for (int64_t group = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib; group < a.num_groups; group += warps) {
+        const int64_t base = group * G;
+        int r[J], T[J], pt0[J], tk[J];
+        float sp[J];
+        bool valid[J], bad[J];
+        int n_fail = 0;
 #pragma unroll
-    for (int b = 0; b <= kMaxM; ++b) {
-        int c = 0;
-        if (b <= M) {
-#pragma unroll
-            for (int j = 0; j < J; ++j) c += __popc(__ballot_sync(0xffffffffu, valid[j] && r[j] == b));
+        for (int j = 0; j < J; ++j) {
+            const int i = lane + 32 * j;
+            valid[j] = i < G;
+            int pt = 0, nt = 1;
+            sp[j] = 0.f;
+            tk[j] = 0;
+            if (valid[j]) {
+                pt = a.pass_turn[base + i];
+                nt = a.num_turns[base + i];
+                if (lexi) {
+                    sp[j] = a.speedup[base + i];
+                    tk[j] = a.ntokens[base + i];
+                }
+            }
+            bad[j] = valid[j] && (pt < 0 || pt > M || nt < 1 || nt > M || (pt >= 1 && pt > nt));
+            // Eq. 1 over first-turn outcomes; a malformed outcome counts as failed.
+            const bool fail1 = valid[j] && (bad[j] || pt != 1);
+            n_fail += __popc(__ballot_sync(0xffffffffu, fail1));
+            pt0[j] = (valid[j] && !bad[j]) ? pt : 0;
+            T[j] = nt;
         }
-        hist[b] = c;
-    }
+        // Eq. 2 (or the recorded gate).
+        const bool gate = a.gate_in ? (a.gate_in[group] != 0) : (a.tau_min <= n_fail && n_fail <= a.tau_max);
 
-    // Eq. 5 from the histogram; Eq. 6; sum of squared net scores (exact).
-    int d[J];
-    long long dd = 0;
+        // Tier rule of Sec. 3.2; gated-off groups ran turn 1 only.
 #pragma unroll
-    for (int j = 0; j < J; ++j) {
-        int nw = 0, nb = 0;
-#pragma unroll
-        for (int b = 0; b <= kMaxM; ++b) {
-            nw += (b < r[j]) ? hist[b] : 0;
-            nb += (b > r[j]) ? hist[b] : 0;
-        }
-        d[j] = nw - nb;
-        if (valid[j]) {
-            dd += (long long)d[j] * d[j];
-            const int64_t i = base + lane + 32 * j;
-            if (a.n_worse) a.n_worse[i] = nw;
-            if (a.n_better) a.n_better[i] = nb;
-            if (a.r_out) a.r_out[i] = (uint8_t)r[j];
-            a.T_eff[i] = (uint8_t)T[j];
-        }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) dd += __shfl_xor_sync(0xffffffffu, dd, o);
-
-    // GRPO standardisation.  mean_g R = 0 exactly (every strict pair adds +1
-    // and -1 to the net scores), so A_i = d_i / ((G - 1) (std + eps)) with
-    // (G - 1) std = sqrt(sum d^2 / den), den = G - 1 (unbiased) or G.  fp32
-    // with IEEE division and square root: at most ~3.5 ulp on A.
-    const float gm1 = (float)(G - 1);
-    float inv_scale;
-    if (a.norm == 1 || dd == 0) {
-        inv_scale = 0.f;  // unused, or an all-tied group: no preference signal, A = 0
-    } else {
-        const float den = a.std_unbiased ? gm1 : (float)G;
-        inv_scale = 1.f / (sqrtf((float)dd / den) + gm1 * a.eps_std);
-    }
-#pragma unroll
-    for (int j = 0; j < J; ++j) {
-        if (!valid[j]) continue;
-        const int64_t i = base + lane + 32 * j;
-        const float Ri = (float)d[j] / gm1;                      // Eq. 6, correctly rounded
-        const float Ai = (a.norm == 1) ? Ri : (float)d[j] * inv_scale;
-        if (a.R) a.R[i] = Ri;
-        if (a.A) a.A[i] = Ai;
-        // Sec. 3.3: beta = gamma for A >= 0, else 1; last turn keeps A.
-        const float beta = (Ai >= 0.f) ? a.gamma : 1.f;
-        float* ta = a.turn_adv + i * M;
-        float p = Ai;
-        for (int t = M - 1; t >= 0; --t) {
-            if (t < T[j]) {
-                ta[t] = p;
-                p *= beta;
+        for (int j = 0; j < J; ++j) {
+            const int pt = pt0[j];
+            if (!valid[j] || bad[j]) {
+                r[j] = 0;
+                T[j] = 0;
+            } else if (!gate) {
+                r[j] = (pt == 1) ? M : 0;
+                T[j] = 1;
             } else {
-                ta[t] = 0.f;
+                r[j] = (pt >= 1) ? (M - pt + 1) : 0;
+            }
+            if (bad[j]) flag_status(a.status, 2u);
+        }
+
+        // Eq. 5: N_worse / N_better.
+        int nw[J], nb[J];
+        if constexpr (!lexi) {
+            // The paper's comparator looks only at r: a histogram of tiers via ballots.
+            int hist[kMaxM + 1];
+#pragma unroll
+            for (int b = 0; b <= kMaxM; ++b) {
+                int c = 0;
+                if (b <= M) {
+#pragma unroll
+                    for (int j = 0; j < J; ++j) c += __popc(__ballot_sync(0xffffffffu, valid[j] && r[j] == b));
+                }
+                hist[b] = c;
+            }
+#pragma unroll
+            for (int j = 0; j < J; ++j) {
+                nw[j] = 0;
+                nb[j] = 0;
+#pragma unroll
+                for (int b = 0; b <= kMaxM; ++b) {
+                    nw[j] += (b < r[j]) ? hist[b] : 0;
+                    nb[j] += (b > r[j]) ? hist[b] : 0;
+                }
+            }
+        } else {
+            // Tie-broken comparator: every rollout against every peer, keys
+            // broadcast from the lane that holds them.
+#pragma unroll
+            for (int j = 0; j < J; ++j) nw[j] = nb[j] = 0;
+#pragma unroll
+            for (int sidx = 0; sidx < J; ++sidx) {
+                for (int l = 0; l < 32; ++l) {
+                    const int jj = 32 * sidx + l;
+                    if (jj >= G) break;  // uniform across the warp
+                    const int rj = __shfl_sync(0xffffffffu, r[sidx], l);
+                    const float spj = __shfl_sync(0xffffffffu, sp[sidx], l);
+                    const int tkj = __shfl_sync(0xffffffffu, tk[sidx], l);
+#pragma unroll
+                    for (int q = 0; q < J; ++q) {
+                        if (!valid[q] || lane + 32 * q == jj) continue;
+                        const bool tie_r = r[q] == rj && rj > 0;
+                        nw[q] += (r[q] > rj) || (tie_r && (sp[q] > spj || (sp[q] == spj && tk[q] < tkj)));
+                        nb[q] += (rj > r[q]) || (tie_r && (spj > sp[q] || (spj == sp[q] && tkj < tk[q])));
+                    }
+                }
             }
         }
+
+        // Eq. 6 and the sum of squared net scores (exact).
+        int d[J];
+        long long dd = 0;
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            d[j] = nw[j] - nb[j];
+            if (valid[j]) {
+                dd += (long long)d[j] * d[j];
+                const int64_t i = base + lane + 32 * j;
+                if (a.n_worse) a.n_worse[i] = nw[j];
+                if (a.n_better) a.n_better[i] = nb[j];
+                if (a.r_out) a.r_out[i] = (uint8_t)r[j];
+                a.T_eff[i] = (uint8_t)T[j];
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) dd += __shfl_xor_sync(0xffffffffu, dd, o);
+
+        const float gm1 = (float)(G - 1);
+        const float den = a.std_unbiased ? gm1 : (float)G;
+        float Rv[J], Av[J];
+        if (a.reward == 0) {
+            // GRPO standardisation of the tournament reward.  mean_g R = 0
+            // exactly (every strict pair adds +1 and -1 to the net scores), so
+            // A_i = d_i / ((G - 1)(std + eps)) with (G - 1) std = sqrt(sum d^2 / den).
+            // fp32 with IEEE division and square root: at most ~3.5 ulp on A.
+            float inv_scale = 0.f;  // all-tied group: no preference signal, A = 0
+            if (a.norm == 0 && dd != 0) inv_scale = 1.f / (sqrtf((float)dd / den) + gm1 * a.eps_std);
+#pragma unroll
+            for (int j = 0; j < J; ++j) {
+                Rv[j] = (float)d[j] / gm1;  // correctly rounded
+                Av[j] = (a.norm == 1) ? Rv[j] : (float)d[j] * inv_scale;
+            }
+        } else {
+            // Static-scalar baseline reward, standard GRPO with its own mean.
+            float sum = 0.f, lo = 2.f, hi = -1.f;
+#pragma unroll
+            for (int j = 0; j < J; ++j) {
+                Rv[j] = (r[j] == M) ? 1.f : ((r[j] > 0) ? a.static_c : 0.f);
+                if (valid[j]) {
+                    sum += Rv[j];
+                    lo = fminf(lo, Rv[j]);
+                    hi = fmaxf(hi, Rv[j]);
+                }
+            }
+            const float mean = warp_sum_f(sum) / (float)G;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+                hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+            }
+            float ss = 0.f;
+#pragma unroll
+            for (int j = 0; j < J; ++j)
+                if (valid[j]) ss += (Rv[j] - mean) * (Rv[j] - mean);
+            const float stdv = sqrtf(warp_sum_f(ss) / den);
+#pragma unroll
+            for (int j = 0; j < J; ++j)
+                Av[j] = (a.norm == 1) ? Rv[j] : ((hi == lo) ? 0.f : (Rv[j] - mean) / (stdv + a.eps_std));
+        }
+
+        int nonzero = 0;
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            nonzero += __popc(__ballot_sync(0xffffffffu, valid[j] && Av[j] != 0.f));
+            if (!valid[j]) continue;
+            const int64_t i = base + lane + 32 * j;
+            if (a.R) a.R[i] = Rv[j];
+            if (a.A) a.A[i] = Av[j];
+            // Sec. 3.3: beta = gamma for A >= 0, else 1; last turn keeps A.
+            const float beta = (Av[j] >= 0.f) ? a.gamma : 1.f;
+            float* ta = a.turn_adv + i * M;
+            float p = Av[j];
+            for (int t = M - 1; t >= 0; --t) {
+                if (t < T[j]) {
+                    ta[t] = p;
+                    p *= beta;
+                } else {
+                    ta[t] = 0.f;
+                }
+            }
+        }
+        if (lane == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
+
+        if (a.stats) {  // training-observability counters (Table 5, Sec. 4.2)
+            int first = 0, later = 0, failed_on = 0, turns = 0;
+            int by_turn[kMaxM];
+#pragma unroll
+            for (int m = 0; m < kMaxM; ++m) by_turn[m] = 0;
+#pragma unroll
+            for (int j = 0; j < J; ++j) {
+                const bool ok = valid[j] && !bad[j];
+                const int pt = pt0[j];
+                first += __popc(__ballot_sync(0xffffffffu, ok && pt == 1));
+                later += __popc(__ballot_sync(0xffffffffu, ok && gate && pt >= 2));
+                failed_on += __popc(__ballot_sync(0xffffffffu, ok && gate && pt != 1));
+                int tsum = valid[j] ? T[j] : 0;
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) tsum += __shfl_xor_sync(0xffffffffu, tsum, o);
+                turns += tsum;
+#pragma unroll
+                for (int m = 1; m < kMaxM; ++m)
+                    by_turn[m] += __popc(__ballot_sync(0xffffffffu, ok && gate && pt == m + 1));
+            }
+            if (lane == 0) {
+                long long* c = sst[wib];
+                c[0] += 1;
+                c[1] += gate;
+                c[2] += G;
+                c[3] += nonzero;
+                c[4] += first;
+                c[5] += later;
+                c[6] += (later > 0);
+                c[7] += failed_on;
+                c[8] += turns;
+                c[9] += first;
+#pragma unroll
+                for (int m = 1; m < kMaxM; ++m) c[9 + m] += by_turn[m];
+            }
+            __syncwarp();
+        }
     }
-    if (lane == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
+
+    if (a.stats) {
+        __syncthreads();
+        if (threadIdx.x < kNumStats) {
+            long long v = 0;
+            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) v += sst[w][threadIdx.x];
+            if (v) atomicAdd(reinterpret_cast<unsigned long long*>(a.stats) + threadIdx.x, (unsigned long long)v);
+        }
+    }
 }
 
 template <int J>
 cudaError_t launch_rank_j(const RankArgs& a, cudaStream_t s) {
     const int warps = 8;
-    const int64_t blocks = ((int64_t)a.num_groups + warps - 1) / warps;
-    rank_adv_kernel<J><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
+    int64_t blocks = ((int64_t)a.num_groups + warps - 1) / warps;
+    // With counters, fewer blocks loop over the groups: one atomic set per block.
+    if (a.stats) blocks = std::min<int64_t>(blocks, (int64_t)device_sm_count() * 16);
+    if (a.cmp == 1) rank_adv_kernel<J, true><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
+    else rank_adv_kernel<J, false><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -32,6 +32,8 @@ LEAP_CMP_PAPER = 0
 LEAP_CMP_LEXI = 1
 LEAP_ADVNORM_GRPO_STD = 0
 LEAP_ADVNORM_NONE = 1
+LEAP_REWARD_RANK = 0
+LEAP_REWARD_STATIC = 1
 LEAP_AGG_SEQ_MEAN_TOKEN_MEAN = 0
 LEAP_AGG_TOKEN_MEAN = 1
 LEAP_LOSS_ACCUMULATE = 1
@@ -58,7 +60,15 @@ class RankParams(ctypes.Structure):
     _fields_ = [("num_groups", ctypes.c_int32), ("G", ctypes.c_int32), ("M", ctypes.c_int32),
                 ("tau_min", ctypes.c_int32), ("tau_max", ctypes.c_int32), ("gamma", ctypes.c_float),
                 ("eps_std", ctypes.c_float), ("cmp", ctypes.c_int32), ("norm", ctypes.c_int32),
-                ("std_unbiased", ctypes.c_int32)]
+                ("std_unbiased", ctypes.c_int32), ("reward", ctypes.c_int32), ("static_c", ctypes.c_float)]
+
+
+class RankStats(ctypes.Structure):
+    _fields_ = [("groups", ctypes.c_int64), ("gated_groups", ctypes.c_int64), ("rollouts", ctypes.c_int64),
+                ("nonzero_adv_rollouts", ctypes.c_int64), ("first_turn_passes", ctypes.c_int64),
+                ("later_passes", ctypes.c_int64), ("groups_with_recovery", ctypes.c_int64),
+                ("failed_first_turn_in_gated", ctypes.c_int64), ("total_turns", ctypes.c_int64),
+                ("passes_by_turn", ctypes.c_int64 * 8)]
 
 
 class LossParams(ctypes.Structure):
@@ -93,7 +103,7 @@ def lib() -> ctypes.CDLL:
     L.leap_get_device_status.restype = S
     L.leap_get_device_status.argtypes = [ctypes.POINTER(ctypes.c_uint32), _P]
     L.leap_group_rank_advantages.restype = S
-    L.leap_group_rank_advantages.argtypes = [ctypes.POINTER(RankParams)] + [_P] * 14
+    L.leap_group_rank_advantages.argtypes = [ctypes.POINTER(RankParams)] + [_P] * 15
     L.leap_rollout_token_counts.restype = S
     L.leap_rollout_token_counts.argtypes = [_I64, _I32, _I32, _P, _P, _P, _I32, _P, _P, _P, _P]
     L.leap_scatter_turn_advantages.restype = S
@@ -164,7 +174,7 @@ def leap_get_device_status(stream=None) -> int:
 def leap_group_rank_advantages(pass_turn, num_turns, *, G, M, tau_min=0, tau_max=None, gamma=1.0,
                                eps_std=1e-6, norm=LEAP_ADVNORM_GRPO_STD, std_unbiased=True,
                                cmp=LEAP_CMP_PAPER, speedup=None, ntokens=None, gate_in=None, out=None,
-                               stream=None):
+                               reward=LEAP_REWARD_RANK, static_c=0.5, stats=None, stream=None):
     """pass_turn, num_turns: int8 [num_groups * G].  Returns a dict of output tensors."""
     n = pass_turn.numel()
     if n % G:
@@ -177,11 +187,13 @@ def leap_group_rank_advantages(pass_turn, num_turns, *, G, M, tau_min=0, tau_max
                    n_worse=_empty(n, torch.int32, pass_turn), n_better=_empty(n, torch.int32, pass_turn),
                    R=_empty(n, torch.float32, pass_turn), A=_empty(n, torch.float32, pass_turn),
                    turn_adv=_empty(n * M, torch.float32, pass_turn), T_eff=_empty(n, torch.uint8, pass_turn))
-    p = RankParams(num_groups, G, M, tau_min, tau_max, gamma, eps_std, cmp, norm, 1 if std_unbiased else 0)
+    p = RankParams(num_groups, G, M, tau_min, tau_max, gamma, eps_std, cmp, norm, 1 if std_unbiased else 0,
+                   reward, static_c)
     st = lib().leap_group_rank_advantages(
         ctypes.byref(p), _ptr(pass_turn), _ptr(num_turns), _ptr(speedup), _ptr(ntokens), _ptr(gate_in),
         _ptr(out.get("gate")), _ptr(out.get("r")), _ptr(out.get("n_worse")), _ptr(out.get("n_better")),
-        _ptr(out.get("R")), _ptr(out.get("A")), _ptr(out["turn_adv"]), _ptr(out["T_eff"]), _stream(stream))
+        _ptr(out.get("R")), _ptr(out.get("A")), _ptr(out["turn_adv"]), _ptr(out["T_eff"]), _ptr(stats),
+        _stream(stream))
     _check(st, "leap_group_rank_advantages")
     return out
 
@@ -381,3 +393,15 @@ def leap_fused_lmhead_logprobs(hidden, W, ids, old_logp, adv, w, *, eps_low=0.2,
                                           _ptr(workspace), workspace.numel(), _ptr(stats), _stream(stream))
     _check(st, "leap_fused_lmhead_logprobs")
     return dict(loss=loss, logp=logp, lse=lse, ell=ell, dhidden=dhidden)
+
+
+def rank_stats_tensor(device):
+    """Zeroed device buffer laid out as leap_rank_stats_t (the counters accumulate)."""
+    return torch.zeros(ctypes.sizeof(RankStats), dtype=torch.uint8, device=device)
+
+
+def read_rank_stats(t) -> dict:
+    s = RankStats.from_buffer_copy(bytes(t.cpu().numpy().tobytes()))
+    d = {k: getattr(s, k) for k, _ in RankStats._fields_ if k != "passes_by_turn"}
+    d["passes_by_turn"] = list(s.passes_by_turn)
+    return d

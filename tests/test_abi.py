@@ -43,14 +43,20 @@ def test_host_argument_checks_need_no_gpu():
     """Invalid arguments are rejected on the host before any CUDA call."""
     from paper_2608_01804_gb300 import leap as L
     lib = L.lib()
-    p = L.RankParams(1, 1, 2, 0, 1, 0.9, 1e-6, 0, 0, 1)       # G = 1: Eq. 6 divides by G - 1
-    assert lib.leap_group_rank_advantages(ctypes.byref(p), *([None] * 13), None) == L.LEAP_ERR_INVALID_ARG
-    p = L.RankParams(1, 8, 9, 0, 1, 0.9, 1e-6, 0, 0, 1)       # M > 8
-    assert lib.leap_group_rank_advantages(ctypes.byref(p), *([None] * 13), None) == L.LEAP_ERR_INVALID_ARG
-    p = L.RankParams(1, 8, 2, 5, 3, 0.9, 1e-6, 0, 0, 1)       # tau_min > tau_max
-    assert lib.leap_group_rank_advantages(ctypes.byref(p), *([None] * 13), None) == L.LEAP_ERR_INVALID_ARG
-    p = L.RankParams(1, 8, 2, 0, 8, 1.5, 1e-6, 0, 0, 1)       # gamma > 1
-    assert lib.leap_group_rank_advantages(ctypes.byref(p), *([None] * 13), None) == L.LEAP_ERR_INVALID_ARG
+    p = L.RankParams(1, 1, 2, 0, 1, 0.9, 1e-6, 0, 0, 1, 0, 0.5)       # G = 1: Eq. 6 divides by G - 1
+    assert lib.leap_group_rank_advantages(ctypes.byref(p), *([None] * 14), None) == L.LEAP_ERR_INVALID_ARG
+    p = L.RankParams(1, 8, 9, 0, 1, 0.9, 1e-6, 0, 0, 1, 0, 0.5)       # M > 8
+    assert lib.leap_group_rank_advantages(ctypes.byref(p), *([None] * 14), None) == L.LEAP_ERR_INVALID_ARG
+    p = L.RankParams(1, 8, 2, 5, 3, 0.9, 1e-6, 0, 0, 1, 0, 0.5)       # tau_min > tau_max
+    assert lib.leap_group_rank_advantages(ctypes.byref(p), *([None] * 14), None) == L.LEAP_ERR_INVALID_ARG
+    p = L.RankParams(1, 8, 2, 0, 8, 1.5, 1e-6, 0, 0, 1, 0, 0.5)       # gamma > 1
+    assert lib.leap_group_rank_advantages(ctypes.byref(p), *([None] * 14), None) == L.LEAP_ERR_INVALID_ARG
+    p = L.RankParams(1, 8, 2, 0, 8, 0.9, 1e-6, 0, 0, 1, 0, 1.5)       # static_c > 1
+    assert lib.leap_group_rank_advantages(ctypes.byref(p), *([None] * 14), None) == L.LEAP_ERR_INVALID_ARG
+    p = L.RankParams(1, 8, 2, 0, 8, 0.9, 1e-6, 1, 0, 1, 0, 0.5)       # LEXI without speedup / tokens
+    pt = ctypes.c_void_p(256)
+    assert lib.leap_group_rank_advantages(ctypes.byref(p), pt, pt, None, None, None, None, None, None, None,
+                                          None, None, pt, pt, None, None) == L.LEAP_ERR_INVALID_ARG
     # ld not a multiple of 8 / misaligned logits.
     assert lib.leap_token_logprobs(ctypes.c_void_p(16), 1001, ctypes.c_void_p(16), 4, 1000, 1.0,
                                    ctypes.c_void_p(16), None, None) == L.LEAP_ERR_INVALID_ARG

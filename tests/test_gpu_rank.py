@@ -115,3 +115,83 @@ def test_empty_and_gamma_one():
     A = gpu["A"].cpu().numpy()
     for i in range(ta.shape[0]):
         assert np.all(ta[i, :T[i]] == A[i]) and np.all(ta[i, T[i]:] == 0)
+
+
+# ---- extensions: tie-broken comparator, static-scalar baseline, counters ----
+
+def test_lexi_tournament_stress_full_size():
+    """65,536 groups x 64 with ~10% exact duplicate tuples: the tie-broken
+    tournament, bit-exact."""
+    pt, nt, sp, tok = synth.tournament_outcomes()
+    G, M = 64, 3
+    L = leap()
+    gpu = L.leap_group_rank_advantages(to_dev(pt, torch.int8), to_dev(nt, torch.int8), G=G, M=M, tau_min=50,
+                                       tau_max=56, gamma=0.9, cmp=L.LEAP_CMP_LEXI,
+                                       speedup=to_dev(sp, torch.float32), ntokens=to_dev(tok, torch.int32))
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, 50, 56, 0.9, cmp=O.CMP_LEXI,
+                            speedup=sp.reshape(-1, G), ntokens=tok.reshape(-1, G))
+    _compare(gpu, orc, M)
+    assert np.any(orc["n_worse"] + orc["n_better"] < G - 1)   # exact ties occurred
+
+
+@pytest.mark.parametrize("G,M", [(8, 2), (64, 3), (100, 4), (1024, 3)])
+def test_lexi_group_sizes(G, M):
+    rng = np.random.default_rng(G + M)
+    groups = max(1, 2048 // G)
+    n = groups * G
+    nt = rng.integers(1, M + 1, size=n).astype(np.int8)
+    pt = np.minimum(np.where(rng.random(n) < 0.6, rng.integers(1, M + 1, size=n), 0), nt).astype(np.int8)
+    sp = rng.choice([0.5, 1.0, 2.0], size=n).astype(np.float32)
+    tok = rng.choice([128, 256], size=n).astype(np.int32)
+    L = leap()
+    gpu = L.leap_group_rank_advantages(to_dev(pt, torch.int8), to_dev(nt, torch.int8), G=G, M=M, tau_max=G,
+                                       gamma=0.8, cmp=L.LEAP_CMP_LEXI, speedup=to_dev(sp, torch.float32),
+                                       ntokens=to_dev(tok, torch.int32))
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, 0, G, 0.8, cmp=O.CMP_LEXI,
+                            speedup=sp.reshape(-1, G), ntokens=tok.reshape(-1, G))
+    _compare(gpu, orc, M)
+
+
+@pytest.mark.parametrize("c,eps", [(0.5, 1e-6), (0.2, 0.0), (1.0, 1e-6)])
+def test_static_reward_baseline(c, eps):
+    b = synth.multiturn_dcp_batch(seed=9)
+    L = leap()
+    gpu = L.leap_group_rank_advantages(to_dev(b.pass_turn, torch.int8), to_dev(b.num_turns, torch.int8), G=b.G,
+                                       M=b.M, tau_max=b.G, gamma=0.9, gate_in=to_dev(b.gate_in, torch.uint8),
+                                       reward=L.LEAP_REWARD_STATIC, static_c=c, eps_std=eps)
+    orc = O.rank_advantages(b.pass_turn.reshape(-1, b.G), b.num_turns.reshape(-1, b.G), b.M, 0, b.G, 0.9,
+                            eps_std=eps, gate_in=b.gate_in, reward=O.REWARD_STATIC, static_c=c)
+    np.testing.assert_array_equal(gpu["n_worse"].cpu().numpy(), orc["n_worse"].reshape(-1))
+    np.testing.assert_allclose(gpu["R"].cpu().numpy(), orc["R"].reshape(-1), rtol=0, atol=1e-7)
+    assert np.max(np.abs(gpu["A"].cpu().numpy() - orc["A"].reshape(-1))) <= TOL_ADV
+    ta = gpu["turn_adv"].cpu().numpy().reshape(-1, b.M)
+    assert np.max(np.abs(ta - orc["turn_adv"].reshape(-1, b.M))) <= TOL_ADV
+
+
+@pytest.mark.parametrize("maker,tau", [(synth.multiturn_dcp_batch, (8, 15)), (synth.tiny_batch, (3, 6))])
+def test_rank_stats_match_oracle(maker, tau):
+    b = maker()
+    L = leap()
+    st = L.rank_stats_tensor("cuda")
+    gpu = L.leap_group_rank_advantages(to_dev(b.pass_turn, torch.int8), to_dev(b.num_turns, torch.int8), G=b.G,
+                                       M=b.M, tau_min=tau[0], tau_max=tau[1], gamma=0.9, stats=st)
+    orc = O.rank_advantages(b.pass_turn.reshape(-1, b.G), b.num_turns.reshape(-1, b.G), b.M, tau[0], tau[1], 0.9)
+    exp = O.rank_stats(orc, b.pass_turn.reshape(-1, b.G), b.M)
+    got = L.read_rank_stats(st)
+    assert got == exp
+    # accumulate: a second call doubles every counter
+    L.leap_group_rank_advantages(to_dev(b.pass_turn, torch.int8), to_dev(b.num_turns, torch.int8), G=b.G, M=b.M,
+                                 tau_min=tau[0], tau_max=tau[1], gamma=0.9, stats=st)
+    got2 = L.read_rank_stats(st)
+    assert got2["total_turns"] == 2 * exp["total_turns"] and got2["groups"] == 2 * exp["groups"]
+
+
+def test_rank_stats_full_size_tournament():
+    pt, nt, sp, tok = synth.tournament_outcomes()
+    G, M = 64, 3
+    L = leap()
+    st = L.rank_stats_tensor("cuda")
+    L.leap_group_rank_advantages(to_dev(pt, torch.int8), to_dev(nt, torch.int8), G=G, M=M, tau_min=50, tau_max=56,
+                                 gamma=0.9, stats=st)
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, 50, 56, 0.9)
+    assert L.read_rank_stats(st) == O.rank_stats(orc, pt.reshape(-1, G), M)
