@@ -225,3 +225,37 @@ def test_lmhead_dhidden_finite_differences():
             lm = O.lmhead_loss_rows(hm, W, ids, old, adv, w, want_dhidden=False)["loss"]
             fd[k, j] = (lp - lm) / (2 * h)
     np.testing.assert_allclose(out["dhidden"], fd, rtol=0, atol=1e-7)
+
+
+def test_lmhead_dW_finite_differences():
+    """dW = dlogits^T . hidden against central differences of the loss in W,
+    including one masked row (w = 0) and two rows sharing a target id."""
+    rng = np.random.default_rng(12)
+    rows, H, V = 6, 5, 11
+    hidden = rng.normal(size=(rows, H))
+    W = rng.normal(0, 0.5, size=(V, H))
+    ids = rng.integers(0, V, size=rows)
+    ids[3] = ids[1]
+    z = hidden @ W.T
+    _, logp = O.log_softmax_rows(z, ids)
+    old = logp + rng.normal(0, 0.1, size=rows)
+    adv = rng.normal(size=rows)
+    w = np.full(rows, 0.2)
+    w[4] = 0.0
+    out = O.lmhead_loss_rows(hidden, W, ids, old, adv, w, want_dW=True)
+    assert out["dW"].shape == (V, H)
+    h = 1e-6
+    fd = np.zeros_like(W)
+    for v in range(V):
+        for j in range(H):
+            Wp, Wm = W.copy(), W.copy()
+            Wp[v, j] += h
+            Wm[v, j] -= h
+            lp = O.lmhead_loss_rows(hidden, Wp, ids, old, adv, w, want_dhidden=False)["loss"]
+            lm = O.lmhead_loss_rows(hidden, Wm, ids, old, adv, w, want_dhidden=False)["loss"]
+            fd[v, j] = (lp - lm) / (2 * h)
+    np.testing.assert_allclose(out["dW"], fd, rtol=0, atol=1e-7)
+    # Masked rows add nothing: dW over the live rows alone is the same.
+    live = w != 0
+    sub = O.lmhead_loss_rows(hidden[live], W, ids[live], old[live], adv[live], w[live], want_dW=True)
+    np.testing.assert_allclose(sub["dW"], out["dW"], rtol=0, atol=1e-15)
