@@ -65,6 +65,7 @@ def parse_args():
     ap.add_argument("--no-rows", action="store_true", help="skip the per-row measurements")
     ap.add_argument("--lmhead-tokens", type=int, default=0,
                     help="run only the fused lm-head (forward + dhidden) on this many tokens, for profiling captures")
+    ap.add_argument("--lmhead-dw", action="store_true", help="with --lmhead-tokens: also the weight gradient dW")
     ap.add_argument("--prompts", type=int, default=16,
                     help="prompts per rank (16 = the benchmark workload; fewer only for profiling captures)")
     return ap.parse_args()
@@ -351,8 +352,9 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
     old8 += synth.normal(N8, 0.05, 503, device)
     st8 = GrpoStep(lb, V, device, gamma=1.0, tau=(0, lb.G), use_gate_in=False)
     st8.advantages()
-    ws8 = torch.empty(L.leap_fused_lmhead_workspace_size(N8, H, V, True), dtype=torch.uint8, device=device)
+    ws8 = torch.empty(L.leap_fused_lmhead_workspace_size(N8, H, V, True, True), dtype=torch.uint8, device=device)
     dh = torch.empty_like(hidden)
+    dW = torch.empty((V, H), dtype=torch.float32, device=device)
     fwd8 = lambda: L.leap_fused_lmhead_logprobs(hidden, W, ids8, old8, st8.adv, st8.w, want_dhidden=False,
                                                 workspace=ws8)
     full8 = lambda: L.leap_fused_lmhead_logprobs(hidden, W, ids8, old8, st8.adv, st8.w, dhidden=dh, workspace=ws8)
@@ -370,7 +372,24 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
                                                      "achieved_tflops": fl / ms / 1e9,
                                                      "frac": fl / ms / 1e9 / tpeak, "throughput": N8 / (ms / 1e3),
                                                      "unit": "tokens/s", "bound": "tensor"}
-    del hidden, W, dh, ws8, flush_buf
+    grads8 = lambda: L.leap_fused_lmhead_logprobs(hidden, W, ids8, old8, st8.adv, st8.w, dhidden=dh, want_dW=True,
+                                                  dW=dW, workspace=ws8)
+    grads8()
+    ms = _timed_launches(grads8, 3, stream)
+    fl = 8.0 * N8 * V * H
+    rows["fused_lmhead_fwd_dhidden_dW_65536x5120xV"] = {"ms": ms, "algorithmic_flops": fl,
+                                                        "achieved_tflops": fl / ms / 1e9,
+                                                        "frac": fl / ms / 1e9 / tpeak, "throughput": N8 / (ms / 1e3),
+                                                        "unit": "tokens/s", "bound": "tensor"}
+    # The weight-gradient GEMM alone: dW[V x H] += DL[8,192 x V]^T . hidden[8,192 x H].
+    dl8 = synth.normal((8192, V), 1e-3, 505, device, dtype=torch.bfloat16)
+    gw = lambda: L.leap_gemm_bf16_tn_f32(dl8, hidden[:8192], out=dW, accumulate=True)
+    gw()
+    ms = _timed_launches(gw, 5, stream)
+    fl = 2.0 * 8192 * V * H
+    rows["gemm_bf16_tn_f32_Vx5120x8192"] = {"ms": ms, "algorithmic_flops": fl, "achieved_tflops": fl / ms / 1e9,
+                                            "frac": fl / ms / 1e9 / tpeak, "bound": "tensor"}
+    del hidden, W, dh, dW, dl8, ws8, flush_buf
     torch.cuda.synchronize()
     return rows
 
@@ -390,14 +409,17 @@ def lmhead_only(args):
     old = synth.normal(N, 1.0, 503, device) - 12.0
     adv = synth.normal(N, 1.0, 504, device)
     w = torch.full((N,), 1.0 / N, device=device)
-    ws = torch.empty(L.leap_fused_lmhead_workspace_size(N, H, V, True), dtype=torch.uint8, device=device)
+    ws = torch.empty(L.leap_fused_lmhead_workspace_size(N, H, V, True, args.lmhead_dw), dtype=torch.uint8,
+                     device=device)
     dh = torch.empty_like(hidden)
-    run = lambda: L.leap_fused_lmhead_logprobs(hidden, W, ids, old, adv, w, dhidden=dh, workspace=ws)
+    dW = torch.empty((V, H), dtype=torch.float32, device=device) if args.lmhead_dw else None
+    run = lambda: L.leap_fused_lmhead_logprobs(hidden, W, ids, old, adv, w, dhidden=dh, want_dW=args.lmhead_dw,
+                                               dW=dW, workspace=ws)
     for _ in range(args.warmup):
         run()
     ms = _timed_launches(run, args.steps, torch.cuda.current_stream())
-    fl = 6.0 * N * V * H
-    print(json.dumps({"lmhead_tokens": N, "ms": ms, "tflops": fl / ms / 1e9,
+    fl = (8.0 if args.lmhead_dw else 6.0) * N * V * H
+    print(json.dumps({"lmhead_tokens": N, "dW": args.lmhead_dw, "ms": ms, "tflops": fl / ms / 1e9,
                       "frac": fl / ms / 1e9 / measured_tensor_peak()}), flush=True)
 
 

@@ -331,7 +331,9 @@ leap_status_t leap_grpo_loss_bwd(
  * 5. Fused lm-head: token log-probs straight from the hidden states, logits =
  *    hidden . W^T computed tile by tile on the tensor cores (tcgen05) and
  *    reduced in tensor memory, never stored; the same clipped surrogate as
- *    section 4; and the gradient with respect to the hidden states.
+ *    section 4; and its gradients with respect to the hidden states and
+ *    the lm-head weight.  The paper trains the policy through Eq. 3; these
+ *    are that objective's gradients for the last layer, by the chain rule.
  * ------------------------------------------------------------------------ */
 
 /*
@@ -344,27 +346,53 @@ leap_status_t leap_gemm_bf16_nt(const uint16_t* A, int64_t lda, const uint16_t* 
                                 uint16_t* C, int64_t ldc, int32_t M, int32_t N, int32_t K,
                                 void* stream);
 
-/* Bytes of workspace leap_fused_lmhead_logprobs needs (with_dhidden: 0 when
- * dhidden will be NULL).  With dhidden it includes a transposed copy of W
- * (H x V bf16) and one 8,192-token chunk of bf16 dlogits. */
-size_t leap_fused_lmhead_workspace_size(int64_t N, int32_t H, int32_t V, int32_t with_dhidden);
+/*
+ * Weight-gradient GEMM building block: C[M x N] = A^T . B (accumulate == 0)
+ * or C += A^T . B (accumulate != 0), with A bf16 [K x M] and B bf16 [K x N]
+ * row-major (so both operands are read MN-major: the contraction runs over
+ * their rows, e.g. tokens), fp32 accumulation on tcgen05 and an fp32 C
+ * [M x N] with leading dimension ldc.  lda >= M and ldb >= N multiples of 8
+ * elements, ldc >= N a multiple of 4; 16-byte aligned bases.  K == 0 sets
+ * C = 0 (or leaves it unchanged when accumulating).  This is the shape of
+ * dW = dlogits^T . hidden in section 5.
+ */
+leap_status_t leap_gemm_bf16_tn_f32(const uint16_t* A, int64_t lda, const uint16_t* B, int64_t ldb,
+                                    float* C, int64_t ldc, int32_t M, int32_t N, int32_t K,
+                                    int32_t accumulate, void* stream);
+
+/* Gradients the fused lm-head is asked for (the `grads` bit set of
+ * leap_fused_lmhead_workspace_size). */
+#define LEAP_LMHEAD_DHIDDEN 1
+#define LEAP_LMHEAD_DW 2
+
+/* Bytes of workspace leap_fused_lmhead_logprobs needs for the gradients in
+ * `grads` (0: forward only).  Either gradient adds one 8,192-token chunk of
+ * bf16 dlogits (8,192 x V); LEAP_LMHEAD_DHIDDEN adds a transposed copy of W
+ * (H x V bf16). */
+size_t leap_fused_lmhead_workspace_size(int64_t N, int32_t H, int32_t V, int32_t grads);
 
 /*
  * hidden bf16 [N x H] (row-major), W bf16 [V x H] (the lm-head weight,
  * row-major); H % 8 == 0, 16-byte aligned bases.  logits z = hidden . W^T,
  * then exactly leap_grpo_loss_fwd's outputs (loss, logp, lse, ell, stats;
  * ids, old_logp, adv, w as there; params->flags may hold
- * LEAP_LOSS_ACCUMULATE).  If dhidden (bf16 [N x H]) is not NULL it receives
- * d loss / d hidden = dlogits . W, computed from bf16 dlogits of 8,192-token
- * chunks.  workspace: >= leap_fused_lmhead_workspace_size bytes, 256-byte
- * aligned.
+ * LEAP_LOSS_ACCUMULATE).  Gradients of the loss (chain rule through z,
+ * from bf16 dlogits recomputed for 8,192-token chunks):
+ *   dhidden  bf16 [N x H], nullable: d loss / d hidden = dlogits . W;
+ *   dW       fp32 [V x H], nullable, 16-byte aligned: d loss / d W =
+ *            dlogits^T . hidden, summed over all N tokens in fp32 (chunk by
+ *            chunk).  With LEAP_LOSS_ACCUMULATE the sum is added into dW
+ *            (gradient accumulation over micro-batches); otherwise dW is
+ *            overwritten (set to 0 when N == 0).
+ * workspace: >= leap_fused_lmhead_workspace_size(N, H, V, grads) bytes for
+ * the gradients requested, 256-byte aligned.
  */
 leap_status_t leap_fused_lmhead_logprobs(
     const leap_loss_params_t* params,
     const uint16_t* hidden, const uint16_t* W, int64_t N, int32_t H, int32_t V,
     const int32_t* ids, const float* old_logp, const float* adv, const float* w,
     float* loss, float* logp, float* lse, float* ell,
-    uint16_t* dhidden,
+    uint16_t* dhidden, float* dW,
     void* workspace, size_t ws_bytes,
     leap_loss_stats_t* stats,
     void* stream);

@@ -376,7 +376,7 @@ def grpo_loss_rows(z, ids, old_logp, adv, w, eps_low=0.2, eps_high=0.2, inv_temp
 # Fused lm-head variant: logits = hidden . W^T, never stored by the library.
 # ---------------------------------------------------------------------------
 def lmhead_loss_rows(hidden, W, ids, old_logp, adv, w, eps_low=0.2, eps_high=0.2,
-                     inv_temp=1.0, grad_scale=1.0, want_dhidden=True, want_dW=False):
+                     inv_temp=1.0, grad_scale=1.0, want_dhidden=True, want_dW=False, dW_rows=None):
     """The same surrogate on logits z = hidden W^T (fp64), plus its gradients
     with respect to both factors of the product (chain rule through z):
 
@@ -384,9 +384,10 @@ def lmhead_loss_rows(hidden, W, ids, old_logp, adv, w, eps_low=0.2, eps_high=0.2
         dW      = dlogits^T . hidden   [V, H]   (sum over the given rows)
 
     hidden float64 [rows, H], W float64 [V, H].  Returns the grpo_loss_rows dict
-    with 'dhidden' and, if asked, 'dW' added.  Rows with w == 0 have zero
-    dlogits, so they add nothing to dW: dW over a subset of rows that holds
-    every row with w != 0 is dW over all rows.
+    with 'dhidden' and, if asked, 'dW' added; with ``dW_rows`` (vocabulary
+    indices) 'dW' holds only those rows of dW, in that order.  Rows with
+    w == 0 have zero dlogits, so they add nothing to dW: dW over a subset of
+    token rows that holds every row with w != 0 is dW over all rows.
     """
     hidden = np.asarray(hidden, dtype=np.float64)
     W = np.asarray(W, dtype=np.float64)
@@ -396,5 +397,6 @@ def lmhead_loss_rows(hidden, W, ids, old_logp, adv, w, eps_low=0.2, eps_high=0.2
     if want_dhidden:
         out["dhidden"] = out["dlogits"] @ W
     if want_dW:
-        out["dW"] = out["dlogits"].T @ hidden
+        dl = out["dlogits"] if dW_rows is None else out["dlogits"][:, np.asarray(dW_rows)]
+        out["dW"] = dl.T @ hidden
     return out

@@ -2,14 +2,18 @@
 // logits = hidden . W^T are produced 128 x 256 tiles at a time into tensor
 // memory and consumed there, so the [N x V] logits never exist in HBM.
 //
-// One persistent, warp-specialised GEMM kernel (both operands K-major bf16,
-// fp32 accumulation) with three epilogues:
+// One persistent, warp-specialised GEMM kernel (bf16 operands, each either
+// K-major or MN-major in global memory, fp32 accumulation) with four
+// epilogues:
 //   EPI_LSE      online (max, sum of 2^((z - max) c1)) per row over a range
 //                of vocabulary tiles, plus the target logit: the log-sum-exp
 //                partials of the token log-probs;
 //   EPI_DLOGITS  recomputed logits tile -> dlogits = coef (1[v = y] -
 //                softmax) in bf16, into a transient token-chunk buffer;
-//   EPI_STORE    the accumulator as bf16 (dhidden = dlogits . (W^T)^T).
+//   EPI_STORE    the accumulator as bf16 (dhidden = dlogits . (W^T)^T);
+//   EPI_ACC_F32  the accumulator added into (or stored to) an fp32 matrix:
+//                the weight gradient dW = dlogits^T . hidden, summed over
+//                token chunks, with both operands read MN-major.
 // Warp 0 issues TMA tile loads (128-byte swizzle) into a 4-stage shared-memory
 // ring; one thread of warp 1 issues tcgen05.mma (M = 128, N = 256, K = 16)
 // into one of two 256-column fp32 accumulators in tensor memory; warps 2-5
@@ -43,19 +47,28 @@ constexpr int LSE_TILES_PER_UNIT = 8;   // 2,048 vocabulary columns per LSE work
 constexpr int64_t DLOGITS_CHUNK_ROWS = 8192;
 
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1),
-// A and B bf16 (bits 7-9 = 1, 10-12 = 1), both K-major (bits 15, 16 = 0),
-// N >> 3 at bits 17-22, M >> 4 at bits 24-28.
-constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                           ((uint32_t)(BM >> 4) << 24);
+// A and B bf16 (bits 7-9 = 1, 10-12 = 1), A / B major-ness at bits 15 / 16
+// (0 = K-major, 1 = MN-major), N >> 3 at bits 17-22, M >> 4 at bits 24-28.
+template <bool AMN, bool BMN>
+__host__ __device__ constexpr uint32_t idesc() {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((AMN ? 1u : 0u) << 15) | ((BMN ? 1u : 0u) << 16) |
+           ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+}
+// An MN-major operand tile is loaded as 64-element (128-byte) wide column
+// blocks of BK rows each; the blocks sit MN_BLOCK bytes apart in the stage.
+constexpr uint32_t MN_BLOCK = BK * 128;
 
-enum { EPI_STORE = 0, EPI_LSE = 1, EPI_DLOGITS = 2 };
+enum { EPI_STORE = 0, EPI_LSE = 1, EPI_DLOGITS = 2, EPI_ACC_F32 = 3 };
 
 struct GemmArgs {
     int32_t M, N, K;
     int32_t tiles_m, tiles_n, tiles_per_unit, units_n;
     int64_t num_units;
     uint16_t* out;            // STORE / DLOGITS: bf16 [M x ldo]
+    float* outf;              // ACC_F32: fp32 [M x ldo]
     int64_t ldo;
+    int32_t accumulate;       // ACC_F32: add into outf (else overwrite)
+    int32_t n_fastest;        // unit order: 0 = consecutive units walk M, 1 = walk N
     float2* part;             // LSE: (max, sum) per (unit column, row) at [nu * M + row]
     float* zy;                // LSE: target logit per row
     const int32_t* ids;       // LSE / DLOGITS: target id per row
@@ -124,6 +137,25 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
     return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
            ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
+// The same for an MN-major tile: each 128-byte row holds 64 consecutive M (or
+// N) elements of one k, 8-row (8 k) groups are 1024 bytes apart (stride byte
+// offset) and the 64-element column blocks MN_BLOCK bytes apart (leading
+// byte offset).
+__device__ __forceinline__ uint64_t sw128_mn_desc(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)(MN_BLOCK >> 4) << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// Work unit u -> (vocabulary-unit / N-tile group nu, M tile mb).
+__device__ __forceinline__ void unit_coords(const GemmArgs& g, int64_t u, int& nu, int& mb) {
+    if (g.n_fastest) {
+        nu = (int)(u % g.units_n);
+        mb = (int)(u / g.units_n);
+    } else {
+        nu = (int)(u / g.tiles_m);
+        mb = (int)(u % g.tiles_m);
+    }
+}
 
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     uint32_t r[32];
@@ -146,7 +178,7 @@ __device__ __forceinline__ void store_bf16_8(uint16_t* dst, const float* v, int 
     }
 }
 
-template <int EPI>
+template <int EPI, bool AMN, bool BMN>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmArgs g) {
     extern __shared__ uint8_t dsmem[];
@@ -181,15 +213,29 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         if (lane == 0) {
             uint32_t it = 0;
             for (int64_t u = blockIdx.x; u < g.num_units; u += gridDim.x) {
-                const int nu = (int)(u / g.tiles_m), mb = (int)(u % g.tiles_m);
+                int nu, mb;
+                unit_coords(g, u, nu, mb);
                 const int t1 = min(g.tiles_n, (nu + 1) * g.tiles_per_unit);
                 for (int nt = nu * g.tiles_per_unit; nt < t1; ++nt) {
                     for (int kb = 0; kb < nk; ++kb, ++it) {
                         const uint32_t s = it % STAGES;
                         if (it >= STAGES) mbar_wait(&sm.empty[s], ((it / STAGES) - 1) & 1u, g.status, &sm.abort_flag);
                         mbar_arrive_expect_tx(&sm.full[s], STAGE_BYTES);
-                        tma_load_2d(stage0 + s * STAGE_BYTES, &tmA, kb * BK, mb * BM, &sm.full[s]);
-                        tma_load_2d(stage0 + s * STAGE_BYTES + A_TILE, &tmB, kb * BK, nt * BN, &sm.full[s]);
+                        const uint32_t a_dst = stage0 + s * STAGE_BYTES, b_dst = a_dst + A_TILE;
+                        if (AMN) {
+#pragma unroll
+                            for (int j = 0; j < BM / 64; ++j)
+                                tma_load_2d(a_dst + j * MN_BLOCK, &tmA, mb * BM + 64 * j, kb * BK, &sm.full[s]);
+                        } else {
+                            tma_load_2d(a_dst, &tmA, kb * BK, mb * BM, &sm.full[s]);
+                        }
+                        if (BMN) {
+#pragma unroll
+                            for (int j = 0; j < BN / 64; ++j)
+                                tma_load_2d(b_dst + j * MN_BLOCK, &tmB, nt * BN + 64 * j, kb * BK, &sm.full[s]);
+                        } else {
+                            tma_load_2d(b_dst, &tmB, kb * BK, nt * BN, &sm.full[s]);
+                        }
                     }
                 }
             }
@@ -199,7 +245,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         if (lane == 0) {
             uint32_t it = 0, tc = 0;
             for (int64_t u = blockIdx.x; u < g.num_units; u += gridDim.x) {
-                const int nu = (int)(u / g.tiles_m);
+                int nu, mb;
+                unit_coords(g, u, nu, mb);
                 const int t1 = min(g.tiles_n, (nu + 1) * g.tiles_per_unit);
                 for (int nt = nu * g.tiles_per_unit; nt < t1; ++nt, ++tc) {
                     const uint32_t ab = tc & 1u;
@@ -212,8 +259,13 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                         tc_fence_after();
                         const uint32_t a0 = stage0 + s * STAGE_BYTES, b0 = a0 + A_TILE;
 #pragma unroll
-                        for (int k = 0; k < BK / 16; ++k)
-                            umma_bf16(d, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), IDESC, (kb | k) != 0);
+                        for (int k = 0; k < BK / 16; ++k) {
+                            // K = 16 per MMA: 32 bytes along a K-major row, or
+                            // 16 rows (two 1024-byte groups) of an MN-major tile.
+                            const uint64_t da = AMN ? sw128_mn_desc(a0 + k * 2048) : sw128_desc(a0 + k * 32);
+                            const uint64_t db = BMN ? sw128_mn_desc(b0 + k * 2048) : sw128_desc(b0 + k * 32);
+                            umma_bf16(d, da, db, idesc<AMN, BMN>(), (kb | k) != 0);
+                        }
                         umma_commit(&sm.empty[s]);  // the stage is free once these MMAs are done
                     }
                     umma_commit(&sm.acc_full[ab]);
@@ -226,13 +278,14 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         const int rl = ew * 32 + lane;
         uint32_t tc = 0;
         for (int64_t u = blockIdx.x; u < g.num_units; u += gridDim.x) {
-            const int nu = (int)(u / g.tiles_m), mb = (int)(u % g.tiles_m);
+            int nu, mb;
+            unit_coords(g, u, nu, mb);
             const int t1 = min(g.tiles_n, (nu + 1) * g.tiles_per_unit);
             const int64_t row = (int64_t)mb * BM + rl;
             const bool valid = row < g.M;
             int y = -1;
             float rk = 0.f, coef = 0.f;
-            if (valid && EPI != EPI_STORE) y = g.ids[row];
+            if (valid && (EPI == EPI_LSE || EPI == EPI_DLOGITS)) y = g.ids[row];
             if (valid && EPI == EPI_DLOGITS) {
                 rk = g.rowK[row];
                 coef = g.rowcoef[row];
@@ -271,6 +324,29 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                             for (int j = 0; j < 32; ++j)
                                 if (y == col0 + j) zyv = v[j];
                             hasy = true;
+                        }
+                    } else if (EPI == EPI_ACC_F32) {
+                        if (valid) {
+                            float* dst = g.outf + row * g.ldo + col0;
+                            if (col0 + 32 <= g.N) {
+#pragma unroll
+                                for (int q = 0; q < 8; ++q) {
+                                    float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                                    float4* p4 = reinterpret_cast<float4*>(dst + 4 * q);
+                                    if (g.accumulate) {
+                                        const float4 c = *p4;
+                                        o.x += c.x;
+                                        o.y += c.y;
+                                        o.z += c.z;
+                                        o.w += c.w;
+                                    }
+                                    *p4 = o;
+                                }
+                            } else {
+#pragma unroll
+                                for (int j = 0; j < 32; ++j)
+                                    if (col0 + j < g.N) dst[j] = g.accumulate ? dst[j] + v[j] : v[j];
+                            }
                         }
                     } else if (valid) {
                         float o[32];
@@ -383,12 +459,14 @@ bool make_tmap(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int EPI>
+// Tensor maps: a K-major operand [rows x K] is read in boxes of BK x BM (or
+// BN) rows; an MN-major operand [K x rows] in boxes of 64 x BK.
+template <int EPI, bool AMN = false, bool BMN = false>
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, GemmArgs g, cudaStream_t s) {
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [] {
-        attr_err = cudaFuncSetAttribute(tc_gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        attr_err = cudaFuncSetAttribute(tc_gemm_kernel<EPI, AMN, BMN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         (int)GEMM_DYN_SMEM);
     });
     if (attr_err != cudaSuccess) return attr_err;
@@ -399,7 +477,7 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, GemmArgs
     g.num_units = (int64_t)g.tiles_m * g.units_n;
     if (g.num_units == 0) return cudaSuccess;
     const int64_t grid = std::min<int64_t>(g.num_units, device_sm_count());
-    tc_gemm_kernel<EPI><<<(unsigned)grid, GEMM_THREADS, GEMM_DYN_SMEM, s>>>(tmA, tmB, g);
+    tc_gemm_kernel<EPI, AMN, BMN><<<(unsigned)grid, GEMM_THREADS, GEMM_DYN_SMEM, s>>>(tmA, tmB, g);
     return cudaGetLastError();
 }
 
@@ -417,7 +495,7 @@ struct LmheadWorkspace {
     size_t bytes;
 };
 
-LmheadWorkspace lmhead_layout(void* base, int64_t N, int32_t H, int32_t V, bool with_dhidden) {
+LmheadWorkspace lmhead_layout(void* base, int64_t N, int32_t H, int32_t V, bool with_dhidden, bool with_dW) {
     LmheadWorkspace w = {};
     const int64_t tiles_n = ((int64_t)V + BN - 1) / BN;
     const int64_t units_n = (tiles_n + LSE_TILES_PER_UNIT - 1) / LSE_TILES_PER_UNIT;
@@ -435,10 +513,8 @@ LmheadWorkspace lmhead_layout(void* base, int64_t N, int32_t H, int32_t V, bool 
     w.rowcoef = reinterpret_cast<float*>(take(N * sizeof(float)));
     w.loss_ws = take(loss_workspace_bytes(N));
     w.chunk = std::min<int64_t>(N, DLOGITS_CHUNK_ROWS);
-    if (with_dhidden) {
-        w.WT = reinterpret_cast<uint16_t*>(take((size_t)H * ldv * 2));
-        w.DL = reinterpret_cast<uint16_t*>(take((size_t)w.chunk * ldv * 2));
-    }
+    if (with_dhidden) w.WT = reinterpret_cast<uint16_t*>(take((size_t)H * ldv * 2));
+    if (with_dhidden || with_dW) w.DL = reinterpret_cast<uint16_t*>(take((size_t)w.chunk * ldv * 2));
     w.bytes = off;
     return w;
 }
@@ -473,16 +549,46 @@ extern "C" leap_status_t leap_gemm_bf16_nt(const uint16_t* A, int64_t lda, const
     return e == cudaSuccess ? LEAP_OK : LEAP_ERR_CUDA;
 }
 
-extern "C" size_t leap_fused_lmhead_workspace_size(int64_t N, int32_t H, int32_t V, int32_t with_dhidden) {
+extern "C" leap_status_t leap_gemm_bf16_tn_f32(const uint16_t* A, int64_t lda, const uint16_t* B, int64_t ldb,
+                                               float* C, int64_t ldc, int32_t M, int32_t N, int32_t K,
+                                               int32_t accumulate, void* stream) {
+    if (M < 0 || N < 0 || K < 0) return LEAP_ERR_INVALID_ARG;
+    if (M == 0 || N == 0) return LEAP_OK;
+    if (!C || !al16(C) || ldc < N || (ldc & 3)) return LEAP_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (K == 0) {   // an empty sum: C = 0 (or unchanged)
+        if (accumulate) return LEAP_OK;
+        return cudaMemset2DAsync(C, (size_t)ldc * 4, 0, (size_t)N * 4, (size_t)M, s) == cudaSuccess ? LEAP_OK
+                                                                                             : LEAP_ERR_CUDA;
+    }
+    if (!A || !B || !al16(A) || !al16(B)) return LEAP_ERR_INVALID_ARG;
+    if (lda < M || ldb < N || (lda & 7) || (ldb & 7)) return LEAP_ERR_INVALID_ARG;
+    CUtensorMap ta, tb;
+    if (!make_tmap(&ta, A, (uint64_t)M, (uint64_t)K, (uint64_t)lda * 2, BK)) return LEAP_ERR_CUDA;
+    if (!make_tmap(&tb, B, (uint64_t)N, (uint64_t)K, (uint64_t)ldb * 2, BK)) return LEAP_ERR_CUDA;
+    GemmArgs g = {};
+    g.M = M;
+    g.N = N;
+    g.K = K;
+    g.tiles_per_unit = 1;
+    g.outf = C;
+    g.ldo = ldc;
+    g.accumulate = accumulate != 0;
+    g.n_fastest = 1;
+    g.status = nullptr;
+    return launch_gemm<EPI_ACC_F32, true, true>(ta, tb, g, s) == cudaSuccess ? LEAP_OK : LEAP_ERR_CUDA;
+}
+
+extern "C" size_t leap_fused_lmhead_workspace_size(int64_t N, int32_t H, int32_t V, int32_t grads) {
     if (N < 0 || H < 1 || V < 1) return 0;
-    return lmhead_layout(nullptr, N, H, V, with_dhidden != 0).bytes;
+    return lmhead_layout(nullptr, N, H, V, (grads & LEAP_LMHEAD_DHIDDEN) != 0, (grads & LEAP_LMHEAD_DW) != 0).bytes;
 }
 
 extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p, const uint16_t* hidden,
                                                     const uint16_t* W, int64_t N, int32_t H, int32_t V,
                                                     const int32_t* ids, const float* old_logp, const float* adv,
                                                     const float* w, float* loss, float* logp, float* lse, float* ell,
-                                                    uint16_t* dhidden, void* workspace, size_t ws_bytes,
+                                                    uint16_t* dhidden, float* dW, void* workspace, size_t ws_bytes,
                                                     leap_loss_stats_t* stats, void* stream) {
     if (!p || !isfinite(p->eps_low) || !isfinite(p->eps_high) || p->eps_low < 0.f || p->eps_high < 0.f)
         return LEAP_ERR_INVALID_ARG;
@@ -491,9 +597,9 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
     if (N < 0 || N > (int64_t)0x7fffffff || H < 1 || V < 1 || (H & 7) != 0 || !loss) return LEAP_ERR_INVALID_ARG;
     if (N > 0 && (!hidden || !W || !ids || !old_logp || !adv || !w || !al16(hidden) || !al16(W)))
         return LEAP_ERR_INVALID_ARG;
-    if (dhidden && !al16(dhidden)) return LEAP_ERR_INVALID_ARG;
+    if ((dhidden && !al16(dhidden)) || (dW && !al16(dW))) return LEAP_ERR_INVALID_ARG;
     if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return LEAP_ERR_INVALID_ARG;
-    const LmheadWorkspace L = lmhead_layout(workspace, N, H, V, dhidden != nullptr);
+    const LmheadWorkspace L = lmhead_layout(workspace, N, H, V, dhidden != nullptr, dW != nullptr);
     if (ws_bytes < L.bytes) return LEAP_ERR_INVALID_ARG;
     unsigned int* status = device_status_ptr();
     if (!status) return LEAP_ERR_CUDA;
@@ -545,18 +651,25 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
     e = launch_loss_reduce(lws, N, loss, stats, (p->flags & LEAP_LOSS_ACCUMULATE) != 0, s);
     if (e != cudaSuccess) return LEAP_ERR_CUDA;
 
-    if (dhidden && N > 0) {
-        // Backward: dhidden = dlogits . W, through token chunks of transient
-        // bf16 dlogits and a transposed copy of W (both operands K-major).
+    const bool acc = (p->flags & LEAP_LOSS_ACCUMULATE) != 0;
+    if (dW && N == 0 && !acc) {   // an empty sum over tokens
+        if (cudaMemsetAsync(dW, 0, (size_t)V * H * sizeof(float), s) != cudaSuccess) return LEAP_ERR_CUDA;
+    }
+    if ((dhidden || dW) && N > 0) {
+        // Backward through token chunks of transient bf16 dlogits:
+        //   dhidden_chunk = DL . W      (K = V; DL and a transposed copy of W, both K-major)
+        //   dW += DL^T . hidden_chunk   (K = chunk tokens; DL and hidden read MN-major)
         const int64_t ldv = ((int64_t)V + 7) & ~int64_t(7);
-        dim3 tgrid((unsigned)((V + 31) / 32), (unsigned)((H + 31) / 32));
-        transpose_bf16_kernel<<<tgrid, dim3(32, 8), 0, s>>>(W, L.WT, V, H, ldv);
-        if ((e = cudaGetLastError()) != cudaSuccess) return LEAP_ERR_CUDA;
         CUtensorMap tWT;
-        if (!make_tmap(&tWT, L.WT, (uint64_t)V, (uint64_t)H, (uint64_t)ldv * 2, BN)) return LEAP_ERR_CUDA;
+        if (dhidden) {
+            dim3 tgrid((unsigned)((V + 31) / 32), (unsigned)((H + 31) / 32));
+            transpose_bf16_kernel<<<tgrid, dim3(32, 8), 0, s>>>(W, L.WT, V, H, ldv);
+            if ((e = cudaGetLastError()) != cudaSuccess) return LEAP_ERR_CUDA;
+            if (!make_tmap(&tWT, L.WT, (uint64_t)V, (uint64_t)H, (uint64_t)ldv * 2, BN)) return LEAP_ERR_CUDA;
+        }
         for (int64_t c0 = 0; c0 < N; c0 += L.chunk) {
             const int64_t cr = std::min<int64_t>(L.chunk, N - c0);
-            CUtensorMap tHc, tDL;
+            CUtensorMap tHc;
             if (!make_tmap(&tHc, hidden + c0 * H, (uint64_t)H, (uint64_t)cr, (uint64_t)H * 2, BM)) return LEAP_ERR_CUDA;
             GemmArgs g1 = {};
             g1.M = (int32_t)cr;
@@ -570,15 +683,35 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
             g1.c1 = c1;
             g1.status = status;
             if (launch_gemm<EPI_DLOGITS>(tHc, tW, g1, s) != cudaSuccess) return LEAP_ERR_CUDA;
-            if (!make_tmap(&tDL, L.DL, (uint64_t)V, (uint64_t)cr, (uint64_t)ldv * 2, BM)) return LEAP_ERR_CUDA;
-            GemmArgs g2 = {};
-            g2.M = (int32_t)cr;
-            g2.N = H;
-            g2.K = V;
-            g2.out = dhidden + c0 * H;
-            g2.ldo = H;
-            g2.status = status;
-            if (launch_gemm<EPI_STORE>(tDL, tWT, g2, s) != cudaSuccess) return LEAP_ERR_CUDA;
+            if (dhidden) {
+                CUtensorMap tDL;
+                if (!make_tmap(&tDL, L.DL, (uint64_t)V, (uint64_t)cr, (uint64_t)ldv * 2, BM)) return LEAP_ERR_CUDA;
+                GemmArgs g2 = {};
+                g2.M = (int32_t)cr;
+                g2.N = H;
+                g2.K = V;
+                g2.out = dhidden + c0 * H;
+                g2.ldo = H;
+                g2.status = status;
+                if (launch_gemm<EPI_STORE>(tDL, tWT, g2, s) != cudaSuccess) return LEAP_ERR_CUDA;
+            }
+            if (dW) {
+                CUtensorMap tDLt, tHt;
+                if (!make_tmap(&tDLt, L.DL, (uint64_t)V, (uint64_t)cr, (uint64_t)ldv * 2, BK)) return LEAP_ERR_CUDA;
+                if (!make_tmap(&tHt, hidden + c0 * H, (uint64_t)H, (uint64_t)cr, (uint64_t)H * 2, BK))
+                    return LEAP_ERR_CUDA;
+                GemmArgs g3 = {};
+                g3.M = V;
+                g3.N = H;
+                g3.K = (int32_t)cr;
+                g3.tiles_per_unit = 1;
+                g3.outf = dW;
+                g3.ldo = H;
+                g3.accumulate = (acc || c0 > 0) ? 1 : 0;
+                g3.n_fastest = 1;   // CTAs in flight share dlogits column blocks; hidden stays in L2
+                g3.status = status;
+                if (launch_gemm<EPI_ACC_F32, true, true>(tDLt, tHt, g3, s) != cudaSuccess) return LEAP_ERR_CUDA;
+            }
         }
     }
     return LEAP_OK;

@@ -38,13 +38,15 @@ LEAP_AGG_SEQ_MEAN_TOKEN_MEAN = 0
 LEAP_AGG_TOKEN_MEAN = 1
 LEAP_LOSS_ACCUMULATE = 1
 LEAP_LOSS_SINGLE_READ = 2
+LEAP_LMHEAD_DHIDDEN = 1
+LEAP_LMHEAD_DW = 2
 
 # Every symbol include/leap.h declares.
 EXPORTS = (
     "leap_status_string", "leap_version", "leap_get_device_status",
     "leap_group_rank_advantages", "leap_rollout_token_counts", "leap_scatter_turn_advantages",
     "leap_token_logprobs", "leap_grpo_loss_workspace_size", "leap_grpo_loss_fwd", "leap_grpo_loss_bwd",
-    "leap_grpo_loss_fwd_noalloc", "leap_gemm_bf16_nt", "leap_fused_lmhead_workspace_size",
+    "leap_grpo_loss_fwd_noalloc", "leap_gemm_bf16_nt", "leap_gemm_bf16_tn_f32", "leap_fused_lmhead_workspace_size",
     "leap_fused_lmhead_logprobs",
 )
 LEAP_NOALLOC_MAX_ROWS = 65536
@@ -121,11 +123,13 @@ def lib() -> ctypes.CDLL:
                                              _P, _P, _P, _P, _P, _P, _P]
     L.leap_gemm_bf16_nt.restype = S
     L.leap_gemm_bf16_nt.argtypes = [_P, _I64, _P, _I64, _P, _I64, _I32, _I32, _I32, _P]
+    L.leap_gemm_bf16_tn_f32.restype = S
+    L.leap_gemm_bf16_tn_f32.argtypes = [_P, _I64, _P, _I64, _P, _I64, _I32, _I32, _I32, _I32, _P]
     L.leap_fused_lmhead_workspace_size.restype = _SZ
     L.leap_fused_lmhead_workspace_size.argtypes = [_I64, _I32, _I32, _I32]
     L.leap_fused_lmhead_logprobs.restype = S
     L.leap_fused_lmhead_logprobs.argtypes = [ctypes.POINTER(LossParams), _P, _P, _I64, _I32, _I32, _P, _P, _P, _P,
-                                             _P, _P, _P, _P, _P, _P, _SZ, _P, _P]
+                                             _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]
     L.leap_grpo_loss_bwd.restype = S
     L.leap_grpo_loss_bwd.argtypes = [ctypes.POINTER(LossParams), _P, _I64, _P, _P, _P, _P, _P, _I64, _I32,
                                      _P, _P]
@@ -359,14 +363,35 @@ def leap_gemm_bf16_nt(A, B, out=None, stream=None):
     return out
 
 
-def leap_fused_lmhead_workspace_size(N, H, V, with_dhidden=True) -> int:
-    return int(lib().leap_fused_lmhead_workspace_size(int(N), int(H), int(V), 1 if with_dhidden else 0))
+def leap_gemm_bf16_tn_f32(A, B, out=None, accumulate=False, stream=None):
+    """out[M x N] (+)= A[K x M]^T . B[K x N] (bf16 in, fp32 accumulation on tcgen05, fp32 out)."""
+    pa, lda = _bf16_2d(A, "A")
+    pb, ldb = _bf16_2d(B, "B")
+    K, M = A.shape
+    N = B.shape[1]
+    if B.shape[0] != K:
+        raise ValueError("contracted dimensions differ")
+    if out is None:   # rows padded to a multiple of 4 elements (16 bytes), returned as an [M x N] view
+        out = torch.empty((M, (N + 3) // 4 * 4), dtype=torch.float32, device=A.device)[:, :N]
+    if out.dtype != torch.float32 or out.dim() != 2 or out.stride(1) != 1:
+        raise ValueError("out must be a 2-D fp32 tensor with contiguous rows")
+    st = lib().leap_gemm_bf16_tn_f32(pa, lda, pb, ldb, ctypes.c_void_p(out.data_ptr()), out.stride(0), M, N, K,
+                                     1 if accumulate else 0, _stream(stream))
+    _check(st, "leap_gemm_bf16_tn_f32")
+    return out
+
+
+def leap_fused_lmhead_workspace_size(N, H, V, with_dhidden=True, with_dW=False) -> int:
+    grads = (LEAP_LMHEAD_DHIDDEN if with_dhidden else 0) | (LEAP_LMHEAD_DW if with_dW else 0)
+    return int(lib().leap_fused_lmhead_workspace_size(int(N), int(H), int(V), grads))
 
 
 def leap_fused_lmhead_logprobs(hidden, W, ids, old_logp, adv, w, *, eps_low=0.2, eps_high=0.2, inv_temp=1.0,
-                               grad_scale=1.0, accumulate=False, want_dhidden=True, loss=None, logp=None, lse=None,
-                               ell=None, dhidden=None, workspace=None, stats=None, stream=None):
-    """Clipped-surrogate loss from hidden states and the lm-head weight (logits never stored)."""
+                               grad_scale=1.0, accumulate=False, want_dhidden=True, want_dW=False, loss=None,
+                               logp=None, lse=None, ell=None, dhidden=None, dW=None, workspace=None, stats=None,
+                               stream=None):
+    """Clipped-surrogate loss from hidden states and the lm-head weight (logits never stored),
+    with the gradients for hidden (bf16) and, if asked, W (fp32; added into `dW` with accumulate)."""
     ph, ldh = _bf16_2d(hidden, "hidden")
     pw, ldw = _bf16_2d(W, "W")
     N, H = hidden.shape
@@ -383,16 +408,23 @@ def leap_fused_lmhead_logprobs(hidden, W, ids, old_logp, adv, w, *, eps_low=0.2,
         dhidden = torch.empty_like(hidden)
     if not want_dhidden:
         dhidden = None
+    if want_dW and dW is None:
+        dW = torch.zeros((V, H), dtype=torch.float32, device=dev)
+    if not want_dW:
+        dW = None
+    if dW is not None and (dW.dtype != torch.float32 or tuple(dW.shape) != (V, H) or not dW.is_contiguous()):
+        raise ValueError("dW must be a contiguous fp32 [V x H] tensor")
     if workspace is None:
-        workspace = torch.empty(max(1, leap_fused_lmhead_workspace_size(N, H, V, want_dhidden)), dtype=torch.uint8,
-                                device=dev)
+        workspace = torch.empty(max(1, leap_fused_lmhead_workspace_size(N, H, V, want_dhidden, want_dW)),
+                                dtype=torch.uint8, device=dev)
     p = LossParams(eps_low, eps_high, inv_temp, grad_scale, LEAP_LOSS_ACCUMULATE if accumulate else 0)
     st = lib().leap_fused_lmhead_logprobs(ctypes.byref(p), ph, pw, N, H, V, _ptr(ids), _ptr(old_logp), _ptr(adv),
                                           _ptr(w), _ptr(loss), _ptr(logp), _ptr(lse), _ptr(ell),
                                           None if dhidden is None else ctypes.c_void_p(dhidden.data_ptr()),
+                                          None if dW is None else ctypes.c_void_p(dW.data_ptr()),
                                           _ptr(workspace), workspace.numel(), _ptr(stats), _stream(stream))
     _check(st, "leap_fused_lmhead_logprobs")
-    return dict(loss=loss, logp=logp, lse=lse, ell=ell, dhidden=dhidden)
+    return dict(loss=loss, logp=logp, lse=lse, ell=ell, dhidden=dhidden, dW=dW)
 
 
 def rank_stats_tensor(device):

@@ -259,3 +259,7 @@ def test_lmhead_dW_finite_differences():
     live = w != 0
     sub = O.lmhead_loss_rows(hidden[live], W, ids[live], old[live], adv[live], w[live], want_dW=True)
     np.testing.assert_allclose(sub["dW"], out["dW"], rtol=0, atol=1e-15)
+    # Selected vocabulary rows of dW are those rows of the whole.
+    pick = [7, 0, ids[1], V - 1]
+    part = O.lmhead_loss_rows(hidden, W, ids, old, adv, w, want_dW=True, dW_rows=pick)
+    np.testing.assert_allclose(part["dW"], out["dW"][pick], rtol=1e-13, atol=1e-15)
