@@ -40,7 +40,7 @@ WORKLOAD = ("single-turn GRPO: 16 prompts x G=8 x 256 token slots = 32,768 rows 
 # dram bytes (read + write) of one fused_loss_kernel launch on this workload: an ncu capture of the
 # kernel built from sources with this SHA-256 on a 4,096-row slice, scaled to the full launch by
 # algorithmic bytes (traffic grows in proportion to them); null once the sources change.
-KNOWN_TRAFFIC = {"src_sha256": "719d7f95fc58e9df03814195268dd11a1da3831c83618cee9e3bb9d4593f1fb1", "bytes_per_launch": 16099568938}
+KNOWN_TRAFFIC = {"src_sha256": "be9e484930faa27e63291a9516bb9ebdf4ba9ebcd9553a739bfc948ec3170203", "bytes_per_launch": 16085954479}
 KERNEL_SOURCES = ("paper_2608_01804_gb300/csrc/logprob_loss.cu", "paper_2608_01804_gb300/csrc/leap_common.cuh",
                   "paper_2608_01804_gb300/csrc/loss_math.cuh")
 
@@ -66,6 +66,8 @@ def parse_args():
     ap.add_argument("--lmhead-tokens", type=int, default=0,
                     help="run only the fused lm-head (forward + dhidden) on this many tokens, for profiling captures")
     ap.add_argument("--lmhead-dw", action="store_true", help="with --lmhead-tokens: also the weight gradient dW")
+    ap.add_argument("--lmhead-vocab", type=int, default=0,
+                    help="with --lmhead-tokens: a smaller vocabulary, only for small profiling captures")
     ap.add_argument("--prompts", type=int, default=16,
                     help="prompts per rank (16 = the benchmark workload; fewer only for profiling captures)")
     return ap.parse_args()
@@ -395,31 +397,32 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
 
 
 def lmhead_only(args):
-    """The fused lm-head alone (H = 5,120, V = 151,936) on --lmhead-tokens tokens:
-    --warmup untimed calls, then --steps timed ones; prints one JSON line."""
+    """The fused lm-head alone (H = 5,120, V = 151,936 unless --lmhead-vocab) on
+    --lmhead-tokens tokens: --warmup untimed calls, then --steps timed ones;
+    prints one JSON line."""
     from paper_2608_01804_gb300 import build
     build.build()
     from paper_2608_01804_gb300 import leap as L
     from paper_2608_01804_gb300 import synth
     device = torch.device("cuda", 0)
-    N, H = args.lmhead_tokens, 5120
+    N, H, Vp = args.lmhead_tokens, 5120, args.lmhead_vocab or V
     hidden = synth.normal((N, H), 1.0, 500, device, dtype=torch.bfloat16)
-    W = synth.normal((V, H), 0.02, 501, device, dtype=torch.bfloat16)
-    ids = synth.token_ids(N, V, 502, device)
+    W = synth.normal((Vp, H), 0.02, 501, device, dtype=torch.bfloat16)
+    ids = synth.token_ids(N, Vp, 502, device)
     old = synth.normal(N, 1.0, 503, device) - 12.0
     adv = synth.normal(N, 1.0, 504, device)
     w = torch.full((N,), 1.0 / N, device=device)
-    ws = torch.empty(L.leap_fused_lmhead_workspace_size(N, H, V, True, args.lmhead_dw), dtype=torch.uint8,
+    ws = torch.empty(L.leap_fused_lmhead_workspace_size(N, H, Vp, True, args.lmhead_dw), dtype=torch.uint8,
                      device=device)
     dh = torch.empty_like(hidden)
-    dW = torch.empty((V, H), dtype=torch.float32, device=device) if args.lmhead_dw else None
+    dW = torch.empty((Vp, H), dtype=torch.float32, device=device) if args.lmhead_dw else None
     run = lambda: L.leap_fused_lmhead_logprobs(hidden, W, ids, old, adv, w, dhidden=dh, want_dW=args.lmhead_dw,
                                                dW=dW, workspace=ws)
     for _ in range(args.warmup):
         run()
     ms = _timed_launches(run, args.steps, torch.cuda.current_stream())
-    fl = (8.0 if args.lmhead_dw else 6.0) * N * V * H
-    print(json.dumps({"lmhead_tokens": N, "dW": args.lmhead_dw, "ms": ms, "tflops": fl / ms / 1e9,
+    fl = (8.0 if args.lmhead_dw else 6.0) * N * Vp * H
+    print(json.dumps({"lmhead_tokens": N, "vocab": Vp, "dW": args.lmhead_dw, "ms": ms, "tflops": fl / ms / 1e9,
                       "frac": fl / ms / 1e9 / measured_tensor_peak()}), flush=True)
 
 
