@@ -40,7 +40,7 @@ WORKLOAD = ("single-turn GRPO: 16 prompts x G=8 x 256 token slots = 32,768 rows 
 # dram bytes (read + write) of one fused_loss_kernel launch on this workload: an ncu capture of the
 # kernel built from sources with this SHA-256 on a 4,096-row slice, scaled to the full launch by
 # algorithmic bytes (traffic grows in proportion to them); null once the sources change.
-KNOWN_TRAFFIC = {"src_sha256": "be9e484930faa27e63291a9516bb9ebdf4ba9ebcd9553a739bfc948ec3170203", "bytes_per_launch": 16085954479}
+KNOWN_TRAFFIC = {"src_sha256": "634708b2b78fb92d5cbf6f119c583ee880890e4bd4ecc276c344ff60102ebb83", "bytes_per_launch": 16148277750}
 KERNEL_SOURCES = ("paper_2608_01804_gb300/csrc/logprob_loss.cu", "paper_2608_01804_gb300/csrc/leap_common.cuh",
                   "paper_2608_01804_gb300/csrc/loss_math.cuh")
 

@@ -68,6 +68,7 @@ struct RowArgs {
     float* ws_rho;
     uint8_t* ws_flag;
     unsigned int* status;
+    int32_t next_stride;  // fused two-pass kernel: rows between a CTA and the one after it on its SM (0 = none)
 };
 
 // Workspace carve-up of leap_grpo_loss_fwd.

@@ -7,6 +7,10 @@
 //                      dlogits.  2V bytes read per row.
 //   fused_loss_l2_kernel  forward + backward, one CTA per row, the second pass
 //                      over the row served by L2.  2V read + 2V written per row.
+//                      A bulk L2 prefetch puts the whole row's HBM reads in
+//                      flight at once, and the head of the row the next CTA
+//                      on the SM will own is prefetched while this one
+//                      writes, so reads and writes overlap on every SM.
 //   fused_loss_kernel  forward + backward with the row split over a cluster
 //                      of C CTAs that keep their slices in registers and
 //                      exchange one (max, sum) pair through distributed
@@ -387,6 +391,43 @@ __global__ void __launch_bounds__(T + 32, MINB) fused_loss_kernel(RowArgs a, int
 // one row per SM in flight (152 rows, 46 MB at V = 151,936) the second read is
 // an L2 hit: DRAM sees 2V bytes read and 2V written per live row.
 // ---------------------------------------------------------------------------
+#ifndef LEAP_L2_PREFETCH
+#define LEAP_L2_PREFETCH 1
+#endif
+#ifndef LEAP_L2_PF_CHUNK
+#define LEAP_L2_PF_CHUNK 32768
+#endif
+#ifndef LEAP_L2_THREADS
+#define LEAP_L2_THREADS 1024
+#endif
+#ifndef LEAP_L2_U
+#define LEAP_L2_U 4
+#endif
+#ifndef LEAP_L2_MINB
+#define LEAP_L2_MINB 1
+#endif
+#ifndef LEAP_L2_NEXT
+#define LEAP_L2_NEXT 1
+#endif
+#ifndef LEAP_L2_NEXT_BYTES
+#define LEAP_L2_NEXT_BYTES 65536
+#endif
+// Warp-wide: bulk L2 prefetch of the first min(cap, row) bytes of a logits row.
+__device__ __forceinline__ void prefetch_row_l2(const uint16_t* zr, int V, int64_t cap, uint64_t policy, int lane) {
+    int64_t bytes = (int64_t)(V & ~7) * 2;
+    if (bytes > cap) bytes = cap & ~int64_t(15);
+    for (int64_t off = (int64_t)lane * LEAP_L2_PF_CHUNK; off < bytes; off += 32 * LEAP_L2_PF_CHUNK)
+        bulk_prefetch_l2(reinterpret_cast<const char*>(zr) + off,
+                         (uint32_t)(bytes - off < LEAP_L2_PF_CHUNK ? bytes - off : LEAP_L2_PF_CHUNK), policy);
+}
+// The row the CTA after this one on the same SM will own (next_stride rows on),
+// if it is live: prefetch its head so its pass 1 overlaps this CTA's writes.
+__device__ __forceinline__ void prefetch_next_row(const RowArgs& a, int64_t row, uint64_t policy, int lane) {
+    const int64_t nr = row + a.next_stride;
+    if (a.next_stride > 0 && nr < a.N && a.w[nr] != 0.f)
+        prefetch_row_l2(a.logits + nr * a.ld, a.V, LEAP_L2_NEXT_BYTES, policy, lane);
+}
+
 template <int T, int U, int MINB>
 __global__ void __launch_bounds__(T, MINB) fused_loss_l2_kernel(RowArgs a) {
     __shared__ float2 wpart[T / 32];
@@ -401,6 +442,9 @@ __global__ void __launch_bounds__(T, MINB) fused_loss_l2_kernel(RowArgs a) {
     const bool bad = (wk != 0.f) && (id < 0 || id >= V);
     uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
     if (wk == 0.f || bad) {
+#if LEAP_L2_NEXT
+        if (warp == 1) prefetch_next_row(a, row, l2_policy_evict_last(), lane);
+#endif
         for (int64_t vi = t; vi < V8; vi += T) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
         if (t == 0) {
             write_masked_outputs(a, row);
@@ -417,6 +461,11 @@ __global__ void __launch_bounds__(T, MINB) fused_loss_l2_kernel(RowArgs a) {
         A = a.adv[row];
     }
     const uint64_t keep = l2_policy_evict_last();
+#if LEAP_L2_PREFETCH
+    // Put the whole row's HBM reads in flight at once: pass 1 then waits on
+    // L2, not on the few loads each thread can hold in registers.
+    if (warp == 0) prefetch_row_l2(zr, V, (int64_t)1 << 40, keep, lane);
+#endif
     const float c1 = a.inv_temp * kLog2e;
     float m = -INFINITY, s = 0.f;
     for (int64_t v0 = t; v0 < V8; v0 += (int64_t)T * U) {
@@ -450,6 +499,9 @@ __global__ void __launch_bounds__(T, MINB) fused_loss_l2_kernel(RowArgs a) {
         }
     }
     __syncthreads();
+#if LEAP_L2_NEXT
+    if (warp == 1) prefetch_next_row(a, row, keep, lane);
+#endif
     const float K = bc[0], coef = bc[1];
     const uint64_t drop = l2_policy_evict_first();
     const int64_t yv = id >> 3;
@@ -738,7 +790,9 @@ cudaError_t launch_split_bwd(const RowArgs& a, cudaStream_t s) {
 cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s) {
     if (a.N == 0) return cudaSuccess;
     if (!single_read) {
-        fused_loss_l2_kernel<1024, 4, 1><<<(unsigned)a.N, 1024, 0, s>>>(a);
+        RowArgs b = a;
+        b.next_stride = device_sm_count() * LEAP_L2_MINB;
+        fused_loss_l2_kernel<LEAP_L2_THREADS, LEAP_L2_U, LEAP_L2_MINB><<<(unsigned)a.N, LEAP_L2_THREADS, 0, s>>>(b);
         return cudaGetLastError();
     }
     const int64_t V8 = ((int64_t)a.V + 7) >> 3;
