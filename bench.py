@@ -66,6 +66,8 @@ def parse_args():
     ap.add_argument("--lmhead-tokens", type=int, default=0,
                     help="run only the fused lm-head (forward + dhidden) on this many tokens, for profiling captures")
     ap.add_argument("--lmhead-dw", action="store_true", help="with --lmhead-tokens: also the weight gradient dW")
+    ap.add_argument("--rank-only", action="store_true",
+                    help="run only the rank advantages on 65,536 groups x 64 rollouts (M = 3), for profiling captures")
     ap.add_argument("--lmhead-vocab", type=int, default=0,
                     help="with --lmhead-tokens: a smaller vocabulary, only for small profiling captures")
     ap.add_argument("--prompts", type=int, default=16,
@@ -426,6 +428,32 @@ def lmhead_only(args):
                       "frac": fl / ms / 1e9 / measured_tensor_peak()}), flush=True)
 
 
+def rank_only(args):
+    """Rank advantages alone on the tournament workload (65,536 groups x 64
+    rollouts, M = 3): --warmup untimed launches, then --steps timed ones,
+    each after an L2 flush; prints one JSON line."""
+    from paper_2608_01804_gb300 import build
+    build.build()
+    from paper_2608_01804_gb300 import leap as L
+    from paper_2608_01804_gb300 import synth
+    device = torch.device("cuda", 0)
+    pt, nt, _, _ = synth.tournament_outcomes()
+    G, M = 64, 3
+    n = pt.size
+    pt_d = torch.as_tensor(pt).to(device)
+    nt_d = torch.as_tensor(nt).to(device)
+    out = L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=50, tau_max=56, gamma=0.9)
+    fn = lambda: L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=50, tau_max=56, gamma=0.9, out=out)
+    flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    for _ in range(args.warmup):
+        fn()
+    ms = _timed_launches(fn, args.steps, torch.cuda.current_stream(), lambda: flush_buf.fill_(1))
+    rank_bytes = n * (2 + 1 + 4 + 4 + 4 + 4 + 4 * M + 1) + n // G
+    peak, _ = measured_peaks()
+    print(json.dumps({"rank_rollouts": n, "ms": ms, "gbs": rank_bytes / ms / 1e6,
+                      "frac": rank_bytes / ms / 1e6 / peak}), flush=True)
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -433,6 +461,9 @@ def main():
         return
     if args.lmhead_tokens:
         lmhead_only(args)
+        return
+    if args.rank_only:
+        rank_only(args)
         return
     rank, world, local = dist_env()
     torch.cuda.set_device(local)

@@ -1,11 +1,13 @@
 // Rank-based advantages (Sec. 3.1 Eqs. 1-2, Sec. 3.2 Eqs. 4-6 + GRPO step,
 // Sec. 3.3 discount) and the per-token scatter of the turn advantages.
 //
-// One warp per rollout group.  Lane l owns rollouts l, l + 32, ...  Because
-// the paper's comparator looks only at the tier r in [0, M], the O(G^2)
-// tournament of Eq. 5 collapses to a histogram of r: N_worse = #peers with a
-// lower tier, N_better = #peers with a higher tier.  The histogram is built
-// with warp ballots, so the whole group stays in registers.
+// One warp per rollout group.  In the generic kernel lane l owns rollouts
+// l, l + 32, ...; in the pair kernel (the paper's comparator, G even and at
+// most 64) it owns 2l and 2l + 1.  Because the paper's comparator looks only
+// at the tier r in [0, M], the O(G^2) tournament of Eq. 5 collapses to a walk
+// over the M + 1 tiers: N_worse = #peers in lower tiers, N_better = #peers in
+// higher tiers, each tier counted with warp ballots, so the whole group stays
+// in registers.
 #include "leap_common.cuh"
 #include "leap_internal.h"
 
@@ -26,8 +28,141 @@ __device__ __forceinline__ float warp_sum_f(float v) {
 // Per-warp running counters (lane 0), reduced per block then added atomically.
 constexpr int kNumStats = 9 + kMaxM;
 
+// Eq. 6 and the advantage of every rollout the lane holds: the tournament
+// reward with the GRPO step, or the static-scalar baseline reward.
+template <int J>
+__device__ __forceinline__ void group_reward(const RankArgs& a, int G, int M, const int (&d)[J], const int (&r)[J],
+                                             const bool (&valid)[J], int dd, float (&Rv)[J], float (&Av)[J]) {
+    const float gm1 = (float)(G - 1);
+    const float den = a.std_unbiased ? gm1 : (float)G;
+    if (a.reward == 0) {
+        // GRPO standardisation of the tournament reward.  mean_g R = 0
+        // exactly (every strict pair adds +1 and -1 to the net scores), so
+        // A_i = d_i / ((G - 1)(std + eps)) with (G - 1) std = sqrt(sum d^2 / den).
+        // fp32 with IEEE division and square root: at most ~3.5 ulp on A.
+        float inv_scale = 0.f;  // all-tied group: no preference signal, A = 0
+        if (a.norm == 0 && dd != 0) inv_scale = 1.f / (sqrtf((float)dd / den) + gm1 * a.eps_std);
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            Rv[j] = (float)d[j] / gm1;  // correctly rounded
+            Av[j] = (a.norm == 1) ? Rv[j] : (float)d[j] * inv_scale;
+        }
+    } else {
+        // Static-scalar baseline reward, standard GRPO with its own mean.
+        float sum = 0.f, lo = 2.f, hi = -1.f;
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            Rv[j] = (r[j] == M) ? 1.f : ((r[j] > 0) ? a.static_c : 0.f);
+            if (valid[j]) {
+                sum += Rv[j];
+                lo = fminf(lo, Rv[j]);
+                hi = fmaxf(hi, Rv[j]);
+            }
+        }
+        const float mean = warp_sum_f(sum) / (float)G;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+            hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+        }
+        float ss = 0.f;
+#pragma unroll
+        for (int j = 0; j < J; ++j)
+            if (valid[j]) ss += (Rv[j] - mean) * (Rv[j] - mean);
+        const float stdv = sqrtf(warp_sum_f(ss) / den);
+#pragma unroll
+        for (int j = 0; j < J; ++j)
+            Av[j] = (a.norm == 1) ? Rv[j] : ((hi == lo) ? 0.f : (Rv[j] - mean) / (stdv + a.eps_std));
+    }
+}
+
+// Training-observability counters of one group (Table 5, Sec. 4.2), added to
+// the warp's row of shared-memory counters by lane 0.
+template <int J>
+__device__ __forceinline__ void group_stats(long long* cnt, int G, bool gate, const bool (&valid)[J],
+                                            const bool (&bad)[J], const int (&pt0)[J], const int (&T)[J],
+                                            const float (&Av)[J], int lane) {
+    int nonzero = 0, first = 0, later = 0, failed_on = 0, turns = 0;
+    int by_turn[kMaxM];
+#pragma unroll
+    for (int m = 0; m < kMaxM; ++m) by_turn[m] = 0;
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+        const bool ok = valid[j] && !bad[j];
+        const int pt = pt0[j];
+        nonzero += __popc(__ballot_sync(0xffffffffu, valid[j] && Av[j] != 0.f));
+        first += __popc(__ballot_sync(0xffffffffu, ok && pt == 1));
+        later += __popc(__ballot_sync(0xffffffffu, ok && gate && pt >= 2));
+        failed_on += __popc(__ballot_sync(0xffffffffu, ok && gate && pt != 1));
+        int tsum = valid[j] ? T[j] : 0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) tsum += __shfl_xor_sync(0xffffffffu, tsum, o);
+        turns += tsum;
+#pragma unroll
+        for (int m = 1; m < kMaxM; ++m)
+            by_turn[m] += __popc(__ballot_sync(0xffffffffu, ok && gate && pt == m + 1));
+    }
+    if (lane == 0) {
+        long long* c = cnt;
+        c[0] += 1;
+        c[1] += gate;
+        c[2] += G;
+        c[3] += nonzero;
+        c[4] += first;
+        c[5] += later;
+        c[6] += (later > 0);
+        c[7] += failed_on;
+        c[8] += turns;
+        c[9] += first;
+#pragma unroll
+        for (int m = 1; m < kMaxM; ++m) c[9 + m] += by_turn[m];
+    }
+    __syncwarp();
+}
+
+// One rollout's outcome fields: malformed (pass_turn outside [0, M], turns
+// outside [1, M], a pass after the last generated turn) or well formed, and
+// whether it failed its first turn (Eq. 1; a malformed outcome counts as
+// failed).  pt0 is the pass turn with malformed outcomes mapped to 0.
+__device__ __forceinline__ void decode_outcome(int pt, int nt, int M, bool valid, bool& bad, bool& fail1, int& pt0) {
+    bad = valid && (pt < 0 || pt > M || nt < 1 || nt > M || (pt >= 1 && pt > nt));
+    fail1 = valid && (bad || pt != 1);
+    pt0 = (valid && !bad) ? pt : 0;
+}
+
+// Tier rule of Sec. 3.2 (r = M - m + 1 for a pass at turn m, 0 for a fail)
+// and the turns that count; gated-off groups ran turn 1 only.
+__device__ __forceinline__ void tier_rule(int pt, int nt, bool valid, bool bad, bool gate, int M, int& r, int& T) {
+    if (!valid || bad) {
+        r = 0;
+        T = 0;
+    } else if (!gate) {
+        r = (pt == 1) ? M : 0;
+        T = 1;
+    } else {
+        r = (pt >= 1) ? (M - pt + 1) : 0;
+        T = nt;
+    }
+}
+
+// Adds the block's shared-memory counters to the caller's leap_rank_stats_t.
+__device__ __forceinline__ void flush_stats(const RankArgs& a, long long (*sst)[kNumStats]) {
+    __syncthreads();
+    if (threadIdx.x < kNumStats) {
+        long long v = 0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) v += sst[w][threadIdx.x];
+        if (v) atomicAdd(reinterpret_cast<unsigned long long*>(a.stats) + threadIdx.x, (unsigned long long)v);
+    }
+}
+
+#ifndef LEAP_RANK_MINB
+#define LEAP_RANK_MINB 4
+#endif
+#ifndef LEAP_RANK_PAIR_MINB
+#define LEAP_RANK_PAIR_MINB 6
+#endif
 template <int J, bool LEXI>  // rollouts per lane: G <= 32 * J; tie-broken comparator
-__global__ void __launch_bounds__(256) rank_adv_kernel(RankArgs a) {
+__global__ void __launch_bounds__(256, (J <= 2 ? LEAP_RANK_MINB : 1)) rank_adv_kernel(RankArgs a) {
     const int lane = threadIdx.x & 31;
     const int wib = threadIdx.x >> 5;
     const int G = a.G, M = a.M;
@@ -60,56 +195,45 @@ __global__ void __launch_bounds__(256) rank_adv_kernel(RankArgs a) {
                     tk[j] = a.ntokens[base + i];
                 }
             }
-            bad[j] = valid[j] && (pt < 0 || pt > M || nt < 1 || nt > M || (pt >= 1 && pt > nt));
-            // Eq. 1 over first-turn outcomes; a malformed outcome counts as failed.
-            const bool fail1 = valid[j] && (bad[j] || pt != 1);
+            bool fail1;
+            decode_outcome(pt, nt, M, valid[j], bad[j], fail1, pt0[j]);
             n_fail += __popc(__ballot_sync(0xffffffffu, fail1));
-            pt0[j] = (valid[j] && !bad[j]) ? pt : 0;
             T[j] = nt;
         }
         // Eq. 2 (or the recorded gate).
         const bool gate = a.gate_in ? (a.gate_in[group] != 0) : (a.tau_min <= n_fail && n_fail <= a.tau_max);
 
-        // Tier rule of Sec. 3.2; gated-off groups ran turn 1 only.
 #pragma unroll
         for (int j = 0; j < J; ++j) {
-            const int pt = pt0[j];
-            if (!valid[j] || bad[j]) {
-                r[j] = 0;
-                T[j] = 0;
-            } else if (!gate) {
-                r[j] = (pt == 1) ? M : 0;
-                T[j] = 1;
-            } else {
-                r[j] = (pt >= 1) ? (M - pt + 1) : 0;
-            }
+            tier_rule(pt0[j], T[j], valid[j], bad[j], gate, M, r[j], T[j]);
             if (bad[j]) flag_status(a.status, 2u);
         }
 
         // Eq. 5: N_worse / N_better.
         int nw[J], nb[J];
         if constexpr (!lexi) {
-            // The paper's comparator looks only at r: a histogram of tiers via ballots.
-            int hist[kMaxM + 1];
+            // The paper's comparator looks only at r: walk the M + 1 tiers in
+            // order, counting each tier's members with ballots; a rollout of
+            // tier b has `below` peers strictly worse and c - 1 tied.
+            int eq[J];
 #pragma unroll
-            for (int b = 0; b <= kMaxM; ++b) {
+            for (int j = 0; j < J; ++j) nw[j] = eq[j] = 0;
+            int below = 0;
+            for (int b = 0; b <= M; ++b) {
                 int c = 0;
-                if (b <= M) {
 #pragma unroll
-                    for (int j = 0; j < J; ++j) c += __popc(__ballot_sync(0xffffffffu, valid[j] && r[j] == b));
+                for (int j = 0; j < J; ++j) c += __popc(__ballot_sync(0xffffffffu, valid[j] && r[j] == b));
+#pragma unroll
+                for (int j = 0; j < J; ++j) {
+                    if (r[j] == b) {
+                        nw[j] = below;
+                        eq[j] = c;
+                    }
                 }
-                hist[b] = c;
+                below += c;
             }
 #pragma unroll
-            for (int j = 0; j < J; ++j) {
-                nw[j] = 0;
-                nb[j] = 0;
-#pragma unroll
-                for (int b = 0; b <= kMaxM; ++b) {
-                    nw[j] += (b < r[j]) ? hist[b] : 0;
-                    nb[j] += (b > r[j]) ? hist[b] : 0;
-                }
-            }
+            for (int j = 0; j < J; ++j) nb[j] = below - nw[j] - eq[j];  // below == G here
         } else {
             // Tie-broken comparator: every rollout against every peer, keys
             // broadcast from the lane that holds them.
@@ -134,14 +258,14 @@ __global__ void __launch_bounds__(256) rank_adv_kernel(RankArgs a) {
             }
         }
 
-        // Eq. 6 and the sum of squared net scores (exact).
+        // Eq. 6 and the sum of squared net scores (exact: at most G (G - 1)^2 < 2^31).
         int d[J];
-        long long dd = 0;
+        int dd = 0;
 #pragma unroll
         for (int j = 0; j < J; ++j) {
             d[j] = nw[j] - nb[j];
             if (valid[j]) {
-                dd += (long long)d[j] * d[j];
+                dd += d[j] * d[j];
                 const int64_t i = base + lane + 32 * j;
                 if (a.n_worse) a.n_worse[i] = nw[j];
                 if (a.n_better) a.n_better[i] = nb[j];
@@ -149,56 +273,13 @@ __global__ void __launch_bounds__(256) rank_adv_kernel(RankArgs a) {
                 a.T_eff[i] = (uint8_t)T[j];
             }
         }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) dd += __shfl_xor_sync(0xffffffffu, dd, o);
+        dd = __reduce_add_sync(0xffffffffu, dd);
 
-        const float gm1 = (float)(G - 1);
-        const float den = a.std_unbiased ? gm1 : (float)G;
         float Rv[J], Av[J];
-        if (a.reward == 0) {
-            // GRPO standardisation of the tournament reward.  mean_g R = 0
-            // exactly (every strict pair adds +1 and -1 to the net scores), so
-            // A_i = d_i / ((G - 1)(std + eps)) with (G - 1) std = sqrt(sum d^2 / den).
-            // fp32 with IEEE division and square root: at most ~3.5 ulp on A.
-            float inv_scale = 0.f;  // all-tied group: no preference signal, A = 0
-            if (a.norm == 0 && dd != 0) inv_scale = 1.f / (sqrtf((float)dd / den) + gm1 * a.eps_std);
-#pragma unroll
-            for (int j = 0; j < J; ++j) {
-                Rv[j] = (float)d[j] / gm1;  // correctly rounded
-                Av[j] = (a.norm == 1) ? Rv[j] : (float)d[j] * inv_scale;
-            }
-        } else {
-            // Static-scalar baseline reward, standard GRPO with its own mean.
-            float sum = 0.f, lo = 2.f, hi = -1.f;
-#pragma unroll
-            for (int j = 0; j < J; ++j) {
-                Rv[j] = (r[j] == M) ? 1.f : ((r[j] > 0) ? a.static_c : 0.f);
-                if (valid[j]) {
-                    sum += Rv[j];
-                    lo = fminf(lo, Rv[j]);
-                    hi = fmaxf(hi, Rv[j]);
-                }
-            }
-            const float mean = warp_sum_f(sum) / (float)G;
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-                hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-            }
-            float ss = 0.f;
-#pragma unroll
-            for (int j = 0; j < J; ++j)
-                if (valid[j]) ss += (Rv[j] - mean) * (Rv[j] - mean);
-            const float stdv = sqrtf(warp_sum_f(ss) / den);
-#pragma unroll
-            for (int j = 0; j < J; ++j)
-                Av[j] = (a.norm == 1) ? Rv[j] : ((hi == lo) ? 0.f : (Rv[j] - mean) / (stdv + a.eps_std));
-        }
+        group_reward<J>(a, G, M, d, r, valid, dd, Rv, Av);
 
-        int nonzero = 0;
 #pragma unroll
         for (int j = 0; j < J; ++j) {
-            nonzero += __popc(__ballot_sync(0xffffffffu, valid[j] && Av[j] != 0.f));
             if (!valid[j]) continue;
             const int64_t i = base + lane + 32 * j;
             if (a.R) a.R[i] = Rv[j];
@@ -218,59 +299,124 @@ __global__ void __launch_bounds__(256) rank_adv_kernel(RankArgs a) {
         }
         if (lane == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
 
-        if (a.stats) {  // training-observability counters (Table 5, Sec. 4.2)
-            int first = 0, later = 0, failed_on = 0, turns = 0;
-            int by_turn[kMaxM];
-#pragma unroll
-            for (int m = 0; m < kMaxM; ++m) by_turn[m] = 0;
-#pragma unroll
-            for (int j = 0; j < J; ++j) {
-                const bool ok = valid[j] && !bad[j];
-                const int pt = pt0[j];
-                first += __popc(__ballot_sync(0xffffffffu, ok && pt == 1));
-                later += __popc(__ballot_sync(0xffffffffu, ok && gate && pt >= 2));
-                failed_on += __popc(__ballot_sync(0xffffffffu, ok && gate && pt != 1));
-                int tsum = valid[j] ? T[j] : 0;
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) tsum += __shfl_xor_sync(0xffffffffu, tsum, o);
-                turns += tsum;
-#pragma unroll
-                for (int m = 1; m < kMaxM; ++m)
-                    by_turn[m] += __popc(__ballot_sync(0xffffffffu, ok && gate && pt == m + 1));
-            }
-            if (lane == 0) {
-                long long* c = sst[wib];
-                c[0] += 1;
-                c[1] += gate;
-                c[2] += G;
-                c[3] += nonzero;
-                c[4] += first;
-                c[5] += later;
-                c[6] += (later > 0);
-                c[7] += failed_on;
-                c[8] += turns;
-                c[9] += first;
-#pragma unroll
-                for (int m = 1; m < kMaxM; ++m) c[9 + m] += by_turn[m];
-            }
-            __syncwarp();
-        }
+        if (a.stats) group_stats<J>(sst[wib], G, gate, valid, bad, pt0, T, Av, lane);
     }
 
-    if (a.stats) {
-        __syncthreads();
-        if (threadIdx.x < kNumStats) {
-            long long v = 0;
-            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) v += sst[w][threadIdx.x];
-            if (v) atomicAdd(reinterpret_cast<unsigned long long*>(a.stats) + threadIdx.x, (unsigned long long)v);
-        }
-    }
+    if (a.stats) flush_stats(a, sst);
 }
 
+// The common case as its own kernel: the paper's comparator, G even and at
+// most 64, M known at compile time.  Lane l holds rollouts 2l and 2l + 1, so
+// it reads both outcomes with one 2-byte load and writes every output of the
+// pair with one vector store (the turn advantages as M float2), and the tier
+// walk and the discount loops unroll.
+template <int MC>
+__global__ void __launch_bounds__(256, LEAP_RANK_PAIR_MINB) rank_pair_kernel(RankArgs a) {
+    constexpr int J = 2, M = MC;
+    const int lane = threadIdx.x & 31;
+    const int wib = threadIdx.x >> 5;
+    const int G = a.G;
+    const bool own = 2 * lane < G;
+    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    __shared__ long long sst[8][kNumStats];
+    if (a.stats) {
+        for (int k = lane; k < kNumStats; k += 32) sst[wib][k] = 0;
+        __syncwarp();
+    }
+
+    for (int64_t group = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib; group < a.num_groups; group += warps) {
+        const int64_t i0 = group * G + 2 * lane;
+        int pt[J] = {0, 0}, T[J] = {1, 1};
+        if (own) {
+            const unsigned p2 = *reinterpret_cast<const uint16_t*>(a.pass_turn + i0);
+            const unsigned n2 = *reinterpret_cast<const uint16_t*>(a.num_turns + i0);
+            pt[0] = (int8_t)(p2 & 0xffu);
+            pt[1] = (int8_t)(p2 >> 8);
+            T[0] = (int8_t)(n2 & 0xffu);
+            T[1] = (int8_t)(n2 >> 8);
+        }
+        bool valid[J] = {own, own}, bad[J];
+        int pt0[J], r[J];
+        int n_fail = 0;
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            bool fail1;
+            decode_outcome(pt[j], T[j], M, valid[j], bad[j], fail1, pt0[j]);
+            n_fail += __popc(__ballot_sync(0xffffffffu, fail1));
+        }
+        const bool gate = a.gate_in ? (a.gate_in[group] != 0) : (a.tau_min <= n_fail && n_fail <= a.tau_max);
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            tier_rule(pt0[j], T[j], valid[j], bad[j], gate, M, r[j], T[j]);
+            if (bad[j]) flag_status(a.status, 2u);
+        }
+
+        // Eq. 5 for the paper's comparator: the ordered tier walk.
+        int nw[J] = {0, 0}, eq[J] = {0, 0}, below = 0;
+#pragma unroll
+        for (int b = 0; b <= M; ++b) {
+            const int c = __popc(__ballot_sync(0xffffffffu, own && r[0] == b)) +
+                          __popc(__ballot_sync(0xffffffffu, own && r[1] == b));
+#pragma unroll
+            for (int j = 0; j < J; ++j) {
+                if (r[j] == b) {
+                    nw[j] = below;
+                    eq[j] = c;
+                }
+            }
+            below += c;
+        }
+        int nb[J], d[J];
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            nb[j] = below - nw[j] - eq[j];
+            d[j] = nw[j] - nb[j];
+        }
+        const int dd = __reduce_add_sync(0xffffffffu, own ? d[0] * d[0] + d[1] * d[1] : 0);
+
+        float Rv[J], Av[J];
+        group_reward<J>(a, G, M, d, r, valid, dd, Rv, Av);
+
+        if (own) {
+            if (a.n_worse) *reinterpret_cast<int2*>(a.n_worse + i0) = make_int2(nw[0], nw[1]);
+            if (a.n_better) *reinterpret_cast<int2*>(a.n_better + i0) = make_int2(nb[0], nb[1]);
+            if (a.r_out) *reinterpret_cast<uint16_t*>(a.r_out + i0) = (uint16_t)(r[0] | (r[1] << 8));
+            *reinterpret_cast<uint16_t*>(a.T_eff + i0) = (uint16_t)(T[0] | (T[1] << 8));
+            if (a.R) *reinterpret_cast<float2*>(a.R + i0) = make_float2(Rv[0], Rv[1]);
+            if (a.A) *reinterpret_cast<float2*>(a.A + i0) = make_float2(Av[0], Av[1]);
+            // Sec. 3.3: beta = gamma for A >= 0, else 1; the last counted turn keeps A.
+            float tv[J][M];
+#pragma unroll
+            for (int j = 0; j < J; ++j) {
+                const float beta = (Av[j] >= 0.f) ? a.gamma : 1.f;
+                float p = Av[j];
+#pragma unroll
+                for (int t = M - 1; t >= 0; --t) {
+                    tv[j][t] = (t < T[j]) ? p : 0.f;
+                    if (t < T[j]) p *= beta;
+                }
+            }
+            float2* ta = reinterpret_cast<float2*>(a.turn_adv + i0 * M);
+#pragma unroll
+            for (int q = 0; q < M; ++q)
+                ta[q] = make_float2(tv[(2 * q) / M][(2 * q) % M], tv[(2 * q + 1) / M][(2 * q + 1) % M]);
+        }
+        if (lane == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
+
+        if (a.stats) group_stats<J>(sst[wib], G, gate, valid, bad, pt0, T, Av, lane);
+    }
+    if (a.stats) flush_stats(a, sst);
+}
+
+#ifndef LEAP_RANK_BLOCKS_PER_SM
+#define LEAP_RANK_BLOCKS_PER_SM 0
+#endif
 template <int J>
 cudaError_t launch_rank_j(const RankArgs& a, cudaStream_t s) {
     const int warps = 8;
     int64_t blocks = ((int64_t)a.num_groups + warps - 1) / warps;
+    if (LEAP_RANK_BLOCKS_PER_SM > 0)
+        blocks = std::min<int64_t>(blocks, (int64_t)device_sm_count() * LEAP_RANK_BLOCKS_PER_SM);
     // With counters, fewer blocks loop over the groups: one atomic set per block.
     if (a.stats) blocks = std::min<int64_t>(blocks, (int64_t)device_sm_count() * 16);
     if (a.cmp == 1) rank_adv_kernel<J, true><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
@@ -391,10 +537,40 @@ __global__ void __launch_bounds__(256) scatter_kernel(SegArgs a) {
     }
 }
 
+bool aligned_to(const void* p, uintptr_t n) { return (reinterpret_cast<uintptr_t>(p) & (n - 1)) == 0; }
+
+template <int MC>
+cudaError_t launch_pair(const RankArgs& a, cudaStream_t s) {
+    const int warps = 8;
+    int64_t blocks = ((int64_t)a.num_groups + warps - 1) / warps;
+    if (a.stats) blocks = std::min<int64_t>(blocks, (int64_t)device_sm_count() * 16);
+    rank_pair_kernel<MC><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_rank_advantages(const RankArgs& a, cudaStream_t s) {
     if (a.num_groups == 0) return cudaSuccess;
+    // The pair kernel's vector accesses need 2-byte aligned byte arrays and
+    // 8-byte aligned 4-byte arrays (rollout pairs start at even indices).
+    const bool pair = a.cmp == 0 && a.G % 2 == 0 && a.G <= 64 && aligned_to(a.pass_turn, 2) &&
+                      aligned_to(a.num_turns, 2) && aligned_to(a.T_eff, 2) && aligned_to(a.r_out, 2) &&
+                      aligned_to(a.n_worse, 8) && aligned_to(a.n_better, 8) && aligned_to(a.R, 8) &&
+                      aligned_to(a.A, 8) && aligned_to(a.turn_adv, 8);
+    if (pair) {
+        switch (a.M) {
+            case 1: return launch_pair<1>(a, s);
+            case 2: return launch_pair<2>(a, s);
+            case 3: return launch_pair<3>(a, s);
+            case 4: return launch_pair<4>(a, s);
+            case 5: return launch_pair<5>(a, s);
+            case 6: return launch_pair<6>(a, s);
+            case 7: return launch_pair<7>(a, s);
+            case 8: return launch_pair<8>(a, s);
+            default: break;
+        }
+    }
     const int J = (a.G + 31) / 32;
     if (J <= 1) return launch_rank_j<1>(a, s);
     if (J <= 2) return launch_rank_j<2>(a, s);

@@ -195,3 +195,34 @@ def test_rank_stats_full_size_tournament():
                                  gamma=0.9, stats=st)
     orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, 50, 56, 0.9)
     assert L.read_rank_stats(st) == O.rank_stats(orc, pt.reshape(-1, G), M)
+
+
+@pytest.mark.parametrize("G,M", [(64, 3), (16, 2), (2, 8)])
+def test_pair_and_generic_kernels_agree(G, M):
+    """Even G <= 64 with the paper's comparator runs the pair kernel (vector
+    loads and stores); outputs that are not 8-byte aligned send the same call
+    to the generic kernel.  Both equal the oracle and each other, bit for bit."""
+    rng = np.random.default_rng(7 * G + M)
+    groups = 2048 // G + 3
+    n = groups * G
+    nt = rng.integers(1, M + 1, size=n).astype(np.int8)
+    pt = np.minimum(np.where(rng.random(n) < 0.5, rng.integers(1, M + 1, size=n), 0), nt).astype(np.int8)
+    pt[5] = M + 1                                   # one malformed outcome
+    L = leap()
+    dev = torch.device("cuda")
+    pt_d, nt_d = torch.as_tensor(pt, device=dev), torch.as_tensor(nt, device=dev)
+    tau = (G // 4, (3 * G) // 4)
+    L.leap_get_device_status()                      # clears the sticky flags
+    aligned = L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=tau[0], tau_max=tau[1], gamma=0.8)
+    off = lambda k, dt: torch.empty(k + 1, dtype=dt, device=dev)[1:]    # 4-byte offset: generic kernel
+    out = dict(gate=off(groups, torch.uint8), r=off(n, torch.uint8), n_worse=off(n, torch.int32),
+               n_better=off(n, torch.int32), R=off(n, torch.float32), A=off(n, torch.float32),
+               turn_adv=off(n * M, torch.float32), T_eff=off(n, torch.uint8))
+    generic = L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=tau[0], tau_max=tau[1], gamma=0.8,
+                                           out=out)
+    torch.cuda.synchronize()
+    assert L.leap_get_device_status() & L.LEAP_DEV_BAD_OUTCOME
+    for k in aligned:
+        assert torch.equal(aligned[k], generic[k]), k
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, tau[0], tau[1], 0.8)
+    _compare(aligned, orc, M)
