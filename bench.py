@@ -68,6 +68,8 @@ def parse_args():
     ap.add_argument("--lmhead-dw", action="store_true", help="with --lmhead-tokens: also the weight gradient dW")
     ap.add_argument("--rank-only", action="store_true",
                     help="run only the rank advantages on 65,536 groups x 64 rollouts (M = 3), for profiling captures")
+    ap.add_argument("--tokens-only", action="store_true",
+                    help="run only the token counts + scatter on the packed multi-turn batch, for profiling captures")
     ap.add_argument("--lmhead-vocab", type=int, default=0,
                     help="with --lmhead-tokens: a smaller vocabulary, only for small profiling captures")
     ap.add_argument("--prompts", type=int, default=16,
@@ -250,13 +252,23 @@ def reference_arm(args):
     print(json.dumps(line), flush=True)
 
 
-def _timed_launches(fn, reps, stream, flush=None):
+# GPU cycles (~100 us) the stream spins before a short row's start event, so
+# that the row's launches are all queued by the time the device reaches them.
+LEAD_CYCLES = 200000
+
+
+def _timed_launches(fn, reps, stream, flush=None, lead_cycles=0):
     """Average device time of fn() over `reps` launches, each timed with CUDA
-    events on the launching stream; `flush` (untimed) runs before each."""
+    events on the launching stream; `flush` (untimed) runs before each.  With
+    lead_cycles the stream first spins that many GPU cycles (untimed), so every
+    launch of fn() is queued before the start event is reached and the time is
+    the device's, not the host's launch latency."""
     total = 0.0
     for _ in range(reps):
         if flush is not None:
             flush()
+        if lead_cycles:
+            torch.cuda._sleep(lead_cycles)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         fn()
@@ -292,7 +304,7 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
     out = L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=50, tau_max=56, gamma=0.9)
     fn = lambda: L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=50, tau_max=56, gamma=0.9, out=out)
     fn()
-    ms = _timed_launches(fn, reps * 4, stream, flush)
+    ms = _timed_launches(fn, reps * 4, stream, flush, lead_cycles=LEAD_CYCLES)
     rank_bytes = n * (2 + 1 + 4 + 4 + 4 + 4 + 4 * M + 1) + n // G
     rows["rank_advantages_65536x64"] = entry(rank_bytes, ms, n, "rollouts/s")
     del pt_d, nt_d, out
@@ -311,7 +323,7 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
     def tok():
         L.leap_rollout_token_counts(b.N, so, sr, st_, rk["T_eff"], M=b.M, L=Lc, totals=tot)
         L.leap_scatter_turn_advantages(b.N, so, sr, st_, rk["turn_adv"], rk["T_eff"], Lc, tot, M=b.M, adv=adv, w=w)
-    ms = _timed_launches(tok, reps * 4, stream, flush)
+    ms = _timed_launches(tok, reps * 4, stream, flush, lead_cycles=LEAD_CYCLES)
     rows["token_counts_scatter_multiturn_%d_tokens" % b.N] = entry(8 * b.N, ms, b.N, "tokens/s")
     del adv, w
 
@@ -447,11 +459,44 @@ def rank_only(args):
     flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device=device)
     for _ in range(args.warmup):
         fn()
-    ms = _timed_launches(fn, args.steps, torch.cuda.current_stream(), lambda: flush_buf.fill_(1))
+    ms = _timed_launches(fn, args.steps, torch.cuda.current_stream(), lambda: flush_buf.fill_(1),
+                         lead_cycles=LEAD_CYCLES)
     rank_bytes = n * (2 + 1 + 4 + 4 + 4 + 4 + 4 * M + 1) + n // G
     peak, _ = measured_peaks()
     print(json.dumps({"rank_rollouts": n, "ms": ms, "gbs": rank_bytes / ms / 1e6,
                       "frac": rank_bytes / ms / 1e6 / peak}), flush=True)
+
+
+def tokens_only(args):
+    """Per-rollout token counts + per-token scatter alone on the packed
+    multi-turn batch: --warmup untimed calls, then --steps timed ones, each
+    after an L2 flush; prints one JSON line."""
+    from paper_2608_01804_gb300 import build
+    build.build()
+    from paper_2608_01804_gb300 import leap as L
+    from paper_2608_01804_gb300 import synth
+    device = torch.device("cuda", 0)
+    b = synth.multiturn_dcp_batch()
+    pt_d = torch.as_tensor(b.pass_turn).to(device)
+    nt_d = torch.as_tensor(b.num_turns).to(device)
+    rk = L.leap_group_rank_advantages(pt_d, nt_d, G=b.G, M=b.M, tau_min=8, tau_max=15, gamma=0.9)
+    so = torch.as_tensor(b.seg_offsets).to(device)
+    sr = torch.as_tensor(b.seg_rollout).to(device)
+    st_ = torch.as_tensor(b.seg_turn).to(device)
+    Lc, tot = L.leap_rollout_token_counts(b.N, so, sr, st_, rk["T_eff"], M=b.M)
+    adv, w = L.leap_scatter_turn_advantages(b.N, so, sr, st_, rk["turn_adv"], rk["T_eff"], Lc, tot, M=b.M)
+
+    def tok():
+        L.leap_rollout_token_counts(b.N, so, sr, st_, rk["T_eff"], M=b.M, L=Lc, totals=tot)
+        L.leap_scatter_turn_advantages(b.N, so, sr, st_, rk["turn_adv"], rk["T_eff"], Lc, tot, M=b.M, adv=adv, w=w)
+    flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    for _ in range(args.warmup):
+        tok()
+    ms = _timed_launches(tok, args.steps, torch.cuda.current_stream(), lambda: flush_buf.fill_(1),
+                         lead_cycles=LEAD_CYCLES)
+    peak, _ = measured_peaks()
+    print(json.dumps({"tokens": b.N, "segments": int(b.seg_rollout.size), "ms": ms, "gbs": 8 * b.N / ms / 1e6,
+                      "frac": 8 * b.N / ms / 1e6 / peak}), flush=True)
 
 
 def main():
@@ -464,6 +509,9 @@ def main():
         return
     if args.rank_only:
         rank_only(args)
+        return
+    if args.tokens_only:
+        tokens_only(args)
         return
     rank, world, local = dist_env()
     torch.cuda.set_device(local)

@@ -488,10 +488,16 @@ __device__ __forceinline__ float recip_count(double x) {
     return (x < 16777216.0) ? 1.f / (float)x : (float)(1.0 / x);
 }
 
-// One warp per chunk of 32 * kScatterIters consecutive tokens: lane 0 finds
-// the chunk's first segment by binary search, then every lane walks forward
-// through the (non-decreasing) offsets as its tokens advance.
-constexpr int kScatterIters = 8;
+// One warp per chunk of 32 * kScatterIters consecutive tokens.  The warp
+// finds the chunk's first segment with a 32-ary search (each level one round
+// of 32 parallel loads and a ballot, so about log32 S dependent loads instead
+// of log2 S), then every lane walks forward through the (non-decreasing)
+// offsets as its tokens advance, reloading a segment's fields only when it
+// enters a new segment.
+#ifndef LEAP_SCATTER_ITERS
+#define LEAP_SCATTER_ITERS 8
+#endif
+constexpr int kScatterIters = LEAP_SCATTER_ITERS;
 
 __global__ void __launch_bounds__(256) scatter_kernel(SegArgs a) {
     const int64_t nv = a.totals_in[0];
@@ -503,16 +509,24 @@ __global__ void __launch_bounds__(256) scatter_kernel(SegArgs a) {
     const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
     for (int64_t c = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); c < nchunks; c += warps) {
         const int64_t k0 = c * chunk;
+        // Last s with seg_offsets[s] <= k0 (0 if none) within [lo, lo + n).
         int32_t seg = 0;
-        if (lane == 0 && S > 0) {  // last s with seg_offsets[s] <= k0 (0 if none)
-            int32_t lo = 0, hi = S;
-            while (hi - lo > 1) {
-                const int32_t mid = (lo + hi) >> 1;
-                if (a.seg_offsets[mid] <= k0) lo = mid; else hi = mid;
+        if (S > 0) {
+            int32_t lo = 0, n = S;
+            while (n > 1) {
+                const int32_t step = (n + 31) / 32;
+                const bool in = lane * step < n;
+                const bool le = in && a.seg_offsets[lo + lane * step] <= k0;
+                const unsigned m = __ballot_sync(0xffffffffu, le);
+                if (m == 0) break;
+                const int32_t hl = 31 - __clz(m);
+                lo += hl * step;
+                n = min(step, n - hl * step);
             }
             seg = lo;
         }
-        seg = __shfl_sync(0xffffffffu, seg, 0);
+        int32_t cur = -1, clo = 0, chi = 0;
+        float cadv = 0.f, cw = 0.f;
 #pragma unroll 1
         for (int it = 0; it < kScatterIters; ++it) {
             const int64_t k = k0 + it * 32 + lane;
@@ -520,15 +534,26 @@ __global__ void __launch_bounds__(256) scatter_kernel(SegArgs a) {
             float adv = 0.f, w = 0.f;
             if (S > 0) {
                 while (seg + 1 < S && a.seg_offsets[seg + 1] <= k) ++seg;
-                int32_t lo, hi, i, t;
-                if (segment_ok(a, seg, lo, hi, i, t) && k >= lo && k < hi && t >= 0 && t < (int)a.T_eff[i]) {
-                    adv = a.turn_adv[(int64_t)i * a.M + t];
-                    if (a.agg == 1) {
-                        w = nv > 0 ? recip_count((double)nv) : 0.f;
+                if (seg != cur) {   // entering a segment: its fields, advantage and weight
+                    cur = seg;
+                    int32_t i, t;
+                    cadv = cw = 0.f;
+                    chi = clo = 0;
+                    if (segment_ok(a, seg, clo, chi, i, t) && t >= 0 && t < (int)a.T_eff[i]) {
+                        cadv = a.turn_adv[(int64_t)i * a.M + t];
+                        if (a.agg == 1) {
+                            cw = nv > 0 ? recip_count((double)nv) : 0.f;
+                        } else {
+                            const int32_t L = a.L_in[i];
+                            cw = (rv > 0 && L > 0) ? recip_count((double)rv * (double)L) : 0.f;
+                        }
                     } else {
-                        const int32_t L = a.L_in[i];
-                        w = (rv > 0 && L > 0) ? recip_count((double)rv * (double)L) : 0.f;
+                        chi = clo;   // no generated tokens here
                     }
+                }
+                if (k >= clo && k < chi) {
+                    adv = cadv;
+                    w = cw;
                 }
             }
             a.adv_out[k] = adv;
