@@ -252,6 +252,9 @@ def reference_arm(args):
     print(json.dumps(line), flush=True)
 
 
+# Rows per host-to-device chunk of the end-to-end leg (1.24 GB of logits at V = 151,936).
+E2E_CHUNK_ROWS = 4096
+
 # GPU cycles (~100 us) the stream spins before a short row's start event, so
 # that the row's launches are all queued by the time the device reaches them.
 LEAD_CYCLES = 200000
@@ -598,9 +601,10 @@ def main():
         E = max(1, args.e2e_steps)
 
         def e2e_step():
-            for k, t in host.items():
-                dev[k].copy_(t, non_blocking=True)
-            step.run(dev["logits"], dev["ids"], dev["old"], dlogits, pg)
+            for k, t in host.items():      # the small inputs; the logits stream in run_streamed
+                if k != "logits":
+                    dev[k].copy_(t, non_blocking=True)
+            step.run_streamed(host["logits"], dev["ids"], dev["old"], dlogits, chunk_rows=E2E_CHUNK_ROWS, pg=pg)
             loss_host.copy_(step.loss, non_blocking=True)
 
         e2e_step()

@@ -80,5 +80,53 @@ class GrpoStep:
         self.loss_pass(logits, ids, old_logp, dlogits)
         return self.loss
 
+    def run_streamed(self, host_logits, ids, old_logp, dlogits, chunk_rows=4096, pg=None):
+        """The whole pass for a batch whose logits are in pinned host memory.
+
+        Chunks of `chunk_rows` rows go to two device staging buffers on a copy
+        stream while the loss runs on the previous chunk on the current stream
+        (the loss accumulates over chunks with LEAP_LOSS_ACCUMULATE; dlogits
+        rows are written in place), so the host-to-device copy of the logits
+        hides the compute.  ids and old_logp are device tensors of all rows.
+        """
+        if not host_logits.is_pinned():
+            raise ValueError("host_logits must be in pinned host memory")
+        N, ld = host_logits.shape
+        comp = torch.cuda.current_stream(self.dev)
+        cs = self._copy_stream()
+        staging = self._staging(chunk_rows, ld, host_logits.dtype)
+        start = torch.cuda.Event()        # after every earlier use of the staging buffers
+        start.record(comp)
+        cs.wait_event(start)
+        self.advantages(pg)                # overlaps the first chunk's copy
+        free = [None, None]
+        for c, a in enumerate(range(0, N, chunk_rows)):
+            b = min(N, a + chunk_rows)
+            buf = staging[c % 2][:b - a]
+            if free[c % 2] is not None:
+                cs.wait_event(free[c % 2])          # the loss that read this buffer is done
+            with torch.cuda.stream(cs):
+                buf.copy_(host_logits[a:b], non_blocking=True)
+            copied = torch.cuda.Event()
+            copied.record(cs)
+            comp.wait_event(copied)
+            self.loss_pass(buf, ids[a:b], old_logp[a:b], dlogits[a:b], row0=a, accumulate=c > 0)
+            done = torch.cuda.Event()
+            done.record(comp)
+            free[c % 2] = done
+        return self.loss
+
+    def _copy_stream(self):
+        if getattr(self, "_cs", None) is None:
+            self._cs = torch.cuda.Stream(self.dev)
+        return self._cs
+
+    def _staging(self, rows, ld, dtype):
+        key = (rows, ld, dtype)
+        if getattr(self, "_stage_key", None) != key:
+            self._stage = [torch.empty((rows, ld), dtype=dtype, device=self.dev) for _ in range(2)]
+            self._stage_key = key
+        return self._stage
+
     # Kernel launches one run() makes (rank 1, counts 3, scatter 1, loss 1 + reduce 2).
     LAUNCHES_PER_RUN = 8

@@ -127,3 +127,36 @@ def test_multiturn_dcp_workload_chunked():
             check_dlogits_rows(bf16_rows_to_f64(dl[sel]), res, rows)
         total_o += float((out["ell"].double() * w[a0:a1].double()).sum().item())
     assert abs(loss.item() - total_o) <= 1e-5 * abs(total_o) + 1e-9
+
+
+def test_streamed_step_equals_resident_step():
+    """GrpoStep.run_streamed (logits in pinned host memory, copied chunk by
+    chunk on a second stream while the loss runs) gives the same dlogits, bit
+    for bit, as GrpoStep.run on resident logits, and exactly the fp32 sum of
+    the per-chunk losses (each the fixed-order fp64 sum rounded to fp32);
+    ragged last chunk."""
+    from paper_2608_01804_gb300.step import GrpoStep
+    b = synth.single_turn_batch(num_prompts=2)
+    V = 151936
+    z = synth.logits(b.N, V, 3.0, 210, "cuda", spike_frac=0.01)
+    ids = synth.token_ids(b.N, V, 211, "cuda")
+    old = torch_logp(z, ids, V) + synth.normal(b.N, 0.05, 212, "cuda")
+    step = GrpoStep(b, V, "cuda", gamma=1.0, tau=(0, b.G), use_gate_in=False)
+    dl_res = torch.empty_like(z)
+    loss_res = step.run(z, ids, old, dl_res).clone()
+    host = z.cpu().pin_memory()
+    dl_str = torch.full_like(z, 7)
+    loss_str = step.run_streamed(host, ids, old, dl_str, chunk_rows=1500).clone()
+    torch.cuda.synchronize()
+    assert torch.equal(dl_str, dl_res)
+    L = leap()
+    expect = torch.zeros(1, device="cuda")
+    scratch = torch.empty_like(z)
+    for a in range(0, b.N, 1500):
+        e = min(b.N, a + 1500)
+        part = L.leap_grpo_loss_fwd(z[a:e], ids[a:e], old[a:e], step.adv[a:e], step.w[a:e], V=V,
+                                    dlogits=scratch[a:e], want_outputs=False)["loss"]
+        expect = expect + part
+    assert loss_str.item() == expect.item()
+    # The whole-batch loss differs from the chunked one only by the fp32 sum over chunks.
+    assert abs(loss_str.item() - loss_res.item()) <= 4 * 2.0 ** -24 * float(step.w.abs().sum().item()) * 2.0
