@@ -310,7 +310,24 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
     ms = _timed_launches(fn, reps * 4, stream, flush, lead_cycles=LEAD_CYCLES)
     rank_bytes = n * (2 + 1 + 4 + 4 + 4 + 4 + 4 * M + 1) + n // G
     rows["rank_advantages_65536x64"] = entry(rank_bytes, ms, n, "rollouts/s")
-    del pt_d, nt_d, out
+    # The extension modes on the same workload: tie-broken tournament (reads
+    # speedup and tokens too), training counters, static-scalar reward.
+    _, _, sp, tk = synth.tournament_outcomes()
+    sp_d = torch.as_tensor(sp).to(device)
+    tk_d = torch.as_tensor(tk).to(device)
+    stats = L.rank_stats_tensor(device)
+    variants = {
+        "rank_advantages_lexi_65536x64": (dict(cmp=L.LEAP_CMP_LEXI, speedup=sp_d, ntokens=tk_d), 8 * n),
+        "rank_advantages_with_counters_65536x64": (dict(stats=stats), 0),
+        "rank_advantages_static_reward_65536x64": (dict(reward=L.LEAP_REWARD_STATIC, static_c=0.5), 0),
+    }
+    for name, (kw, extra) in variants.items():
+        fv = lambda kw=kw: L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=50, tau_max=56, gamma=0.9,
+                                                        out=out, **kw)
+        fv()
+        ms = _timed_launches(fv, reps * 4, stream, flush, lead_cycles=LEAD_CYCLES)
+        rows[name] = entry(rank_bytes + extra, ms, n, "rollouts/s")
+    del pt_d, nt_d, out, sp_d, tk_d, stats
 
     # a4: per-rollout counts + per-token scatter, packed multi-turn batch.
     b = synth.multiturn_dcp_batch()
