@@ -235,24 +235,76 @@ __global__ void __launch_bounds__(256, (J <= 2 ? LEAP_RANK_MINB : 1)) rank_adv_k
 #pragma unroll
             for (int j = 0; j < J; ++j) nb[j] = below - nw[j] - eq[j];  // below == G here
         } else {
-            // Tie-broken comparator: every rollout against every peer, keys
-            // broadcast from the lane that holds them.
+            // Tie-broken comparator: every rollout against every peer.  The
+            // keys of 32 peers at a time are staged in the warp's slice of
+            // shared memory and read back as broadcasts.
+            __shared__ int4 lkeys[8][32];
 #pragma unroll
             for (int j = 0; j < J; ++j) nw[j] = nb[j] = 0;
+            bool keyed = false;
+            if constexpr (J <= 8) {  // larger groups keep their registers for the peer loop
+                bool nan_key = false;
 #pragma unroll
-            for (int sidx = 0; sidx < J; ++sidx) {
-                for (int l = 0; l < 32; ++l) {
-                    const int jj = 32 * sidx + l;
-                    if (jj >= G) break;  // uniform across the warp
-                    const int rj = __shfl_sync(0xffffffffu, r[sidx], l);
-                    const float spj = __shfl_sync(0xffffffffu, sp[sidx], l);
-                    const int tkj = __shfl_sync(0xffffffffu, tk[sidx], l);
+                for (int j = 0; j < J; ++j) nan_key |= valid[j] && r[j] > 0 && isnan(sp[j]);
+                keyed = !__any_sync(0xffffffffu, nan_key);
+            }
+            if (keyed) {
+                // Without NaN the order is total, so each rollout gets one
+                // 96-bit key that orders exactly as the comparator:
+                // (r, speedup, -tokens) for a pass, 0 for a failure (failures
+                // tie whatever their speedup and tokens).  Strict comparisons
+                // never count a rollout against itself.
+                unsigned long long khi[J];
+                unsigned klo[J];
 #pragma unroll
-                    for (int q = 0; q < J; ++q) {
-                        if (!valid[q] || lane + 32 * q == jj) continue;
-                        const bool tie_r = r[q] == rj && rj > 0;
-                        nw[q] += (r[q] > rj) || (tie_r && (sp[q] > spj || (sp[q] == spj && tk[q] < tkj)));
-                        nb[q] += (rj > r[q]) || (tie_r && (spj > sp[q] || (spj == sp[q] && tkj < tk[q])));
+                for (int j = 0; j < J; ++j) {
+                    const unsigned b = __float_as_uint(sp[j] + 0.f);   // -0 -> +0, equal as floats
+                    const unsigned o = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+                    khi[j] = r[j] > 0 ? (((unsigned long long)r[j] << 32) | o) : 0ull;
+                    klo[j] = r[j] > 0 ? ~((unsigned)tk[j] ^ 0x80000000u) : 0u;
+                }
+#pragma unroll
+                for (int sidx = 0; sidx < J; ++sidx) {
+                    const int npeer = min(32, G - 32 * sidx);  // uniform across the warp
+                    if (npeer <= 0) break;
+                    __syncwarp();
+                    lkeys[wib][lane] = make_int4((int)(unsigned)khi[sidx], (int)(unsigned)(khi[sidx] >> 32),
+                                                 (int)klo[sidx], 0);
+                    __syncwarp();
+#pragma unroll(J >= 16 ? 1 : 4)
+                    for (int l = 0; l < npeer; ++l) {
+                        const int4 kj = lkeys[wib][l];
+                        const unsigned long long hj = ((unsigned long long)(unsigned)kj.y << 32) | (unsigned)kj.x;
+                        const unsigned lj = (unsigned)kj.z;
+#pragma unroll
+                        for (int q = 0; q < J; ++q) {
+                            nw[q] += (khi[q] > hj) || (khi[q] == hj && klo[q] > lj);
+                            nb[q] += (hj > khi[q]) || (hj == khi[q] && lj > klo[q]);
+                        }
+                    }
+                }
+            } else {
+                // A NaN speedup compares false both ways, and G > 256 keeps
+                // the registers: the comparator itself, peer by peer.
+#pragma unroll
+                for (int sidx = 0; sidx < J; ++sidx) {
+                    const int npeer = min(32, G - 32 * sidx);
+                    if (npeer <= 0) break;
+                    __syncwarp();
+                    lkeys[wib][lane] = make_int4(r[sidx], __float_as_int(sp[sidx]), tk[sidx], 0);
+                    __syncwarp();
+                    for (int l = 0; l < npeer; ++l) {
+                        const int4 kj = lkeys[wib][l];
+                        const int rj = kj.x, tkj = kj.z;
+                        const float spj = __int_as_float(kj.y);
+                        const int jj = 32 * sidx + l;
+#pragma unroll
+                        for (int q = 0; q < J; ++q) {
+                            if (!valid[q] || lane + 32 * q == jj) continue;
+                            const bool tie_r = r[q] == rj && rj > 0;
+                            nw[q] += (r[q] > rj) || (tie_r && (sp[q] > spj || (sp[q] == spj && tk[q] < tkj)));
+                            nb[q] += (rj > r[q]) || (tie_r && (spj > sp[q] || (spj == sp[q] && tkj < tk[q])));
+                        }
                     }
                 }
             }

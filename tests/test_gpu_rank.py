@@ -226,3 +226,27 @@ def test_pair_and_generic_kernels_agree(G, M):
         assert torch.equal(aligned[k], generic[k]), k
     orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, tau[0], tau[1], 0.8)
     _compare(aligned, orc, M)
+
+
+@pytest.mark.parametrize("G", [8, 64, 100, 300])
+def test_lexi_special_keys(G):
+    """Tie-breaks on edge values: +0 and -0 speedups (equal), infinities,
+    negative and extreme token counts, and NaN speedups in some groups (a NaN
+    compares false both ways, so those groups take the peer-by-peer path)."""
+    rng = np.random.default_rng(3 * G)
+    groups = max(4, 2048 // G)
+    n = groups * G
+    M = 3
+    nt = rng.integers(1, M + 1, size=n).astype(np.int8)
+    pt = np.minimum(np.where(rng.random(n) < 0.7, rng.integers(1, M + 1, size=n), 0), nt).astype(np.int8)
+    sp = rng.choice(np.array([0.0, -0.0, 1.0, np.inf, -np.inf, 2.5, -3.0], dtype=np.float32), size=n)
+    tok = rng.choice(np.array([0, 1, -5, 2 ** 31 - 1, -2 ** 31, 128], dtype=np.int64), size=n).astype(np.int32)
+    sp[G * 1 + 3] = np.nan                       # group 1 has a NaN
+    sp[G * 2: G * 2 + G // 2] = np.nan           # group 2 half NaN
+    L = leap()
+    gpu = L.leap_group_rank_advantages(to_dev(pt, torch.int8), to_dev(nt, torch.int8), G=G, M=M, tau_max=G,
+                                       gamma=0.8, cmp=L.LEAP_CMP_LEXI, speedup=to_dev(sp, torch.float32),
+                                       ntokens=to_dev(tok, torch.int32))
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, 0, G, 0.8, cmp=O.CMP_LEXI,
+                            speedup=sp.reshape(-1, G), ntokens=tok.reshape(-1, G))
+    _compare(gpu, orc, M)
