@@ -35,8 +35,20 @@ namespace {
 
 constexpr int BM = 128;   // tokens per tile (tensor-memory lanes)
 constexpr int BN = 256;   // columns per tile (accumulator columns)
-constexpr int BK = 64;    // K per stage: one 128-byte swizzle row of bf16
-constexpr int STAGES = 4;
+#ifndef LEAP_TC_BK
+#define LEAP_TC_BK 64
+#endif
+#ifndef LEAP_TC_STAGES
+#define LEAP_TC_STAGES (LEAP_TC_BK == 64 ? 4 : 8)
+#endif
+constexpr int BK = LEAP_TC_BK;  // K per stage: one 128-byte (64) or 64-byte (32) swizzle row of bf16
+constexpr int STAGES = LEAP_TC_STAGES;
+static_assert(BK == 64 || BK == 32, "K-major tiles use the 128- or 64-byte swizzle");
+// K-major tiles: rows of BK bf16 (BK * 2 bytes, the swizzle span), 8-row
+// swizzle atoms KROW_ATOM bytes apart; descriptor swizzle code 2 = 128-byte,
+// 4 = 64-byte.
+constexpr uint32_t KROW_ATOM = 8 * BK * 2;
+constexpr uint64_t KSWZ_CODE = (BK == 64) ? 2 : 4;
 constexpr uint32_t A_TILE = BM * BK * 2;
 constexpr uint32_t B_TILE = BN * BK * 2;
 constexpr uint32_t STAGE_BYTES = A_TILE + B_TILE;
@@ -44,6 +56,15 @@ constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
 constexpr int GEMM_THREADS = 192;       // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr size_t GEMM_DYN_SMEM = (size_t)STAGES * STAGE_BYTES + 1024;
 constexpr int LSE_TILES_PER_UNIT = 8;   // 2,048 vocabulary columns per LSE work unit
+#ifndef LEAP_LSE_GROUP_M
+#define LEAP_LSE_GROUP_M 16  // forward: the 152 CTAs in flight cover 16 hidden tiles x ~10 vocabulary units
+#endif
+#ifndef LEAP_DL_GROUP_M
+#define LEAP_DL_GROUP_M 16  // dlogits chunk: 16 token tiles x ~10 vocabulary tiles in flight
+#endif
+#ifndef LEAP_ST_GROUP_M
+#define LEAP_ST_GROUP_M 8   // dhidden: 8 token tiles x 20 hidden tiles (the whole N) in flight
+#endif
 constexpr int64_t DLOGITS_CHUNK_ROWS = 8192;
 
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1),
@@ -69,6 +90,7 @@ struct GemmArgs {
     int64_t ldo;
     int32_t accumulate;       // ACC_F32: add into outf (else overwrite)
     int32_t n_fastest;        // unit order: 0 = consecutive units walk M, 1 = walk N
+    int32_t group_m;          // with n_fastest == 0 and > 0: M tiles walked in groups of group_m
     float2* part;             // LSE: (max, sum) per (unit column, row) at [nu * M + row]
     float* zy;                // LSE: target logit per row
     const int32_t* ids;       // LSE / DLOGITS: target id per row
@@ -129,13 +151,13 @@ __device__ __forceinline__ void tma_load_2d(uint32_t smem_dst, const CUtensorMap
 }
 
 // Shared-memory matrix descriptor of a K-major tile written by TMA with the
-// 128-byte swizzle: rows of 128 bytes, 8-row groups 1024 bytes apart.
-// Fields: start address >> 4 (bits 0-13), leading byte offset >> 4 (16-29,
-// unused for this layout), stride byte offset >> 4 (32-45), descriptor
-// version 1 (bit 46), swizzle mode 2 = 128-byte (bits 61-63).
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
-           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+// 128-byte (64-byte) swizzle: rows of BK * 2 bytes, 8-row groups KROW_ATOM
+// bytes apart.  Fields: start address >> 4 (bits 0-13), leading byte offset
+// >> 4 (16-29, unused for this layout), stride byte offset >> 4 (32-45),
+// descriptor version 1 (bit 46), swizzle mode (bits 61-63).
+__device__ __forceinline__ uint64_t kmajor_desc(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(KROW_ATOM >> 4) << 32) |
+           ((uint64_t)1 << 46) | (KSWZ_CODE << 61);
 }
 // The same for an MN-major tile: each 128-byte row holds 64 consecutive M (or
 // N) elements of one k, 8-row (8 k) groups are 1024 bytes apart (stride byte
@@ -146,11 +168,22 @@ __device__ __forceinline__ uint64_t sw128_mn_desc(uint32_t saddr) {
            ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
-// Work unit u -> (vocabulary-unit / N-tile group nu, M tile mb).
+// Work unit u -> (vocabulary-unit / N-tile group nu, M tile mb).  Grouped
+// order: group_m consecutive M tiles are walked M-fastest across all N units
+// before the next group, so the CTAs in flight hold few distinct A tiles
+// (reused from L2 across their N tiles) and few distinct B tiles.
 __device__ __forceinline__ void unit_coords(const GemmArgs& g, int64_t u, int& nu, int& mb) {
     if (g.n_fastest) {
         nu = (int)(u % g.units_n);
         mb = (int)(u / g.units_n);
+    } else if (g.group_m > 0) {
+        const int64_t per_group = (int64_t)g.group_m * g.units_n;
+        const int64_t grp = u / per_group;
+        const int m0 = (int)(grp * g.group_m);
+        const int gm = min(g.group_m, g.tiles_m - m0);   // the last group may be short
+        const int64_t local = u - grp * per_group;
+        nu = (int)(local / gm);
+        mb = m0 + (int)(local % gm);
     } else {
         nu = (int)(u / g.tiles_m);
         mb = (int)(u % g.tiles_m);
@@ -262,8 +295,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                         for (int k = 0; k < BK / 16; ++k) {
                             // K = 16 per MMA: 32 bytes along a K-major row, or
                             // 16 rows (two 1024-byte groups) of an MN-major tile.
-                            const uint64_t da = AMN ? sw128_mn_desc(a0 + k * 2048) : sw128_desc(a0 + k * 32);
-                            const uint64_t db = BMN ? sw128_mn_desc(b0 + k * 2048) : sw128_desc(b0 + k * 32);
+                            const uint64_t da = AMN ? sw128_mn_desc(a0 + k * 2048) : kmajor_desc(a0 + k * 32);
+                            const uint64_t db = BMN ? sw128_mn_desc(b0 + k * 2048) : kmajor_desc(b0 + k * 32);
                             umma_bf16(d, da, db, idesc<AMN, BMN>(), (kb | k) != 0);
                         }
                         umma_commit(&sm.empty[s]);  // the stage is free once these MMAs are done
@@ -446,17 +479,27 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 // 2-D bf16 tensor map: `inner` contiguous elements per row, `outer` rows of
 // `row_bytes`, box inner 64 (128 bytes, the swizzle span) x box_outer rows.
-bool make_tmap(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
-               uint32_t box_outer) {
+bool make_tmap_box(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+                   uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swz) {
     auto fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[2] = {inner, outer};
     cuuint64_t strides[1] = {row_bytes};
-    cuuint32_t box[2] = {(cuuint32_t)BK, box_outer};
+    cuuint32_t box[2] = {box_inner, box_outer};
     cuuint32_t es[2] = {1, 1};
     return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+// A K-major operand: `inner` = K contiguous, boxes of BK x box_outer rows.
+bool make_tmap(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+               uint32_t box_outer) {
+    return make_tmap_box(tm, base, inner, outer, row_bytes, BK, box_outer,
+                         BK == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B);
+}
+// An MN-major operand: `inner` = M (or N) contiguous, boxes of 64 x BK rows (128-byte swizzle).
+bool make_tmap_mn(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes) {
+    return make_tmap_box(tm, base, inner, outer, row_bytes, 64, BK, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 // Tensor maps: a K-major operand [rows x K] is read in boxes of BK x BM (or
@@ -544,6 +587,7 @@ extern "C" leap_status_t leap_gemm_bf16_nt(const uint16_t* A, int64_t lda, const
     g.tiles_per_unit = 1;
     g.out = C;
     g.ldo = ldc;
+    g.group_m = LEAP_ST_GROUP_M;
     g.status = nullptr;
     const cudaError_t e = launch_gemm<EPI_STORE>(ta, tb, g, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? LEAP_OK : LEAP_ERR_CUDA;
@@ -564,8 +608,8 @@ extern "C" leap_status_t leap_gemm_bf16_tn_f32(const uint16_t* A, int64_t lda, c
     if (!A || !B || !al16(A) || !al16(B)) return LEAP_ERR_INVALID_ARG;
     if (lda < M || ldb < N || (lda & 7) || (ldb & 7)) return LEAP_ERR_INVALID_ARG;
     CUtensorMap ta, tb;
-    if (!make_tmap(&ta, A, (uint64_t)M, (uint64_t)K, (uint64_t)lda * 2, BK)) return LEAP_ERR_CUDA;
-    if (!make_tmap(&tb, B, (uint64_t)N, (uint64_t)K, (uint64_t)ldb * 2, BK)) return LEAP_ERR_CUDA;
+    if (!make_tmap_mn(&ta, A, (uint64_t)M, (uint64_t)K, (uint64_t)lda * 2)) return LEAP_ERR_CUDA;
+    if (!make_tmap_mn(&tb, B, (uint64_t)N, (uint64_t)K, (uint64_t)ldb * 2)) return LEAP_ERR_CUDA;
     GemmArgs g = {};
     g.M = M;
     g.N = N;
@@ -637,6 +681,7 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
         g.N = V;
         g.K = H;
         g.tiles_per_unit = LSE_TILES_PER_UNIT;
+        g.group_m = LEAP_LSE_GROUP_M;
         g.part = L.part;
         g.zy = L.zy;
         g.ids = ids;
@@ -681,6 +726,7 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
             g1.rowK = L.rowK + c0;
             g1.rowcoef = L.rowcoef + c0;
             g1.c1 = c1;
+            g1.group_m = LEAP_DL_GROUP_M;
             g1.status = status;
             if (launch_gemm<EPI_DLOGITS>(tHc, tW, g1, s) != cudaSuccess) return LEAP_ERR_CUDA;
             if (dhidden) {
@@ -692,13 +738,14 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
                 g2.K = V;
                 g2.out = dhidden + c0 * H;
                 g2.ldo = H;
+                g2.group_m = LEAP_ST_GROUP_M;
                 g2.status = status;
                 if (launch_gemm<EPI_STORE>(tDL, tWT, g2, s) != cudaSuccess) return LEAP_ERR_CUDA;
             }
             if (dW) {
                 CUtensorMap tDLt, tHt;
-                if (!make_tmap(&tDLt, L.DL, (uint64_t)V, (uint64_t)cr, (uint64_t)ldv * 2, BK)) return LEAP_ERR_CUDA;
-                if (!make_tmap(&tHt, hidden + c0 * H, (uint64_t)H, (uint64_t)cr, (uint64_t)H * 2, BK))
+                if (!make_tmap_mn(&tDLt, L.DL, (uint64_t)V, (uint64_t)cr, (uint64_t)ldv * 2)) return LEAP_ERR_CUDA;
+                if (!make_tmap_mn(&tHt, hidden + c0 * H, (uint64_t)H, (uint64_t)cr, (uint64_t)H * 2))
                     return LEAP_ERR_CUDA;
                 GemmArgs g3 = {};
                 g3.M = V;
