@@ -40,7 +40,7 @@ WORKLOAD = ("single-turn GRPO: 16 prompts x G=8 x 256 token slots = 32,768 rows 
 # dram bytes (read + write) of one fused_loss_kernel launch on this workload: an ncu capture of the
 # kernel built from sources with this SHA-256 on a 4,096-row slice, scaled to the full launch by
 # algorithmic bytes (traffic grows in proportion to them); null once the sources change.
-KNOWN_TRAFFIC = {"src_sha256": "634708b2b78fb92d5cbf6f119c583ee880890e4bd4ecc276c344ff60102ebb83", "bytes_per_launch": 16148277750}
+KNOWN_TRAFFIC = {"src_sha256": "dd6abfb01c786daecf9c2edd643c0c975f83c4f1853f28f40cc6542a9f802688", "bytes_per_launch": 16323515669}
 KERNEL_SOURCES = ("paper_2608_01804_gb300/csrc/logprob_loss.cu", "paper_2608_01804_gb300/csrc/leap_common.cuh",
                   "paper_2608_01804_gb300/csrc/loss_math.cuh")
 
@@ -601,7 +601,7 @@ def main():
     if KNOWN_TRAFFIC and KNOWN_TRAFFIC.get("src_sha256") == _src_sha():
         traffic = KNOWN_TRAFFIC["bytes_per_launch"]
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                "traffic": traffic, "kernel": "fused_loss_l2_kernel<1024,4,1> (+2 reduce launches in the timing)",
+                "traffic": traffic, "kernel": "fused_loss_l2_kernel<1024,4,1,persistent> (+2 reduce launches in the timing)",
                 "algorithmic_bytes_per_launch": alg_bytes, "launch_ms": loss_ms, "peak_source": peak_kind}
 
     # End to end through the same public calls, inputs copied from pinned host memory every step.

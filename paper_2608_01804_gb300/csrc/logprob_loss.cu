@@ -5,12 +5,13 @@
 //   row_stream_kernel  one pass over each logits row with an online
 //                      (max, sum) -> log-probs, or the loss forward without
 //                      dlogits.  2V bytes read per row.
-//   fused_loss_l2_kernel  forward + backward, one CTA per row, the second pass
-//                      over the row served by L2.  2V read + 2V written per row.
-//                      A bulk L2 prefetch puts the whole row's HBM reads in
-//                      flight at once, and the head of the row the next CTA
-//                      on the SM will own is prefetched while this one
-//                      writes, so reads and writes overlap on every SM.
+//   fused_loss_l2_kernel  forward + backward, one persistent CTA per SM taking
+//                      rows round-robin, two passes per row, the second
+//                      served by L2.  2V read + 2V written per row.  A bulk
+//                      L2 prefetch puts the whole row's HBM reads in flight
+//                      at once, and the head of the CTA's next row is
+//                      prefetched while this one writes, so reads and writes
+//                      overlap on every SM.
 //   fused_loss_kernel  forward + backward with the row split over a cluster
 //                      of C CTAs that keep their slices in registers and
 //                      exchange one (max, sum) pair through distributed
@@ -428,11 +429,9 @@ __device__ __forceinline__ void prefetch_next_row(const RowArgs& a, int64_t row,
         prefetch_row_l2(a.logits + nr * a.ld, a.V, LEAP_L2_NEXT_BYTES, policy, lane);
 }
 
-template <int T, int U, int MINB>
-__global__ void __launch_bounds__(T, MINB) fused_loss_l2_kernel(RowArgs a) {
-    __shared__ float2 wpart[T / 32];
-    __shared__ float bc[2];
-    const int64_t row = blockIdx.x;
+// One row of the fused two-pass forward + backward, by the whole CTA.
+template <int T, int U>
+__device__ __forceinline__ void l2_row(const RowArgs& a, const int64_t row, float2* wpart, float* bc) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int V = a.V;
     const int64_t V8 = ((int64_t)V + 7) >> 3;
@@ -526,6 +525,23 @@ __global__ void __launch_bounds__(T, MINB) fused_loss_l2_kernel(RowArgs a) {
             const int64_t vi = v0 + (int64_t)u * T;
             if (vi < V8) store_vec(drow, vi, dlogit8(x[u], c1, K, coef, vi == yv ? ylane : -1), V8, tailn);
         }
+    }
+}
+
+#ifndef LEAP_L2_PERSISTENT
+#define LEAP_L2_PERSISTENT 1
+#endif
+// PERSIST: one CTA per SM walks rows blockIdx.x, + gridDim.x, ... with no CTA
+// launch between rows (the round-robin spreads masked and live rows evenly);
+// otherwise one CTA per row.
+template <int T, int U, int MINB, bool PERSIST>
+__global__ void __launch_bounds__(T, MINB) fused_loss_l2_kernel(RowArgs a) {
+    __shared__ float2 wpart[T / 32];
+    __shared__ float bc[2];
+    if (PERSIST) {
+        for (int64_t row = blockIdx.x; row < a.N; row += gridDim.x) l2_row<T, U>(a, row, wpart, bc);
+    } else {
+        l2_row<T, U>(a, blockIdx.x, wpart, bc);
     }
 }
 
@@ -791,8 +807,17 @@ cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s
     if (a.N == 0) return cudaSuccess;
     if (!single_read) {
         RowArgs b = a;
-        b.next_stride = device_sm_count() * LEAP_L2_MINB;
-        fused_loss_l2_kernel<LEAP_L2_THREADS, LEAP_L2_U, LEAP_L2_MINB><<<(unsigned)a.N, LEAP_L2_THREADS, 0, s>>>(b);
+        const int64_t resident = (int64_t)device_sm_count() * LEAP_L2_MINB;
+        if (LEAP_L2_PERSISTENT) {
+            const int64_t grid = std::min<int64_t>(a.N, resident);
+            b.next_stride = (int32_t)grid;   // exactly this CTA's next row
+            fused_loss_l2_kernel<LEAP_L2_THREADS, LEAP_L2_U, LEAP_L2_MINB, true>
+                <<<(unsigned)grid, LEAP_L2_THREADS, 0, s>>>(b);
+        } else {
+            b.next_stride = (int32_t)resident;   // about the row the next CTA on this SM takes
+            fused_loss_l2_kernel<LEAP_L2_THREADS, LEAP_L2_U, LEAP_L2_MINB, false>
+                <<<(unsigned)a.N, LEAP_L2_THREADS, 0, s>>>(b);
+        }
         return cudaGetLastError();
     }
     const int64_t V8 = ((int64_t)a.V + 7) >> 3;
