@@ -70,6 +70,8 @@ def parse_args():
                     help="run only the rank advantages on 65,536 groups x 64 rollouts (M = 3), for profiling captures")
     ap.add_argument("--tokens-only", action="store_true",
                     help="run only the token counts + scatter on the packed multi-turn batch, for profiling captures")
+    ap.add_argument("--logprobs-only", action="store_true",
+                    help="run only the log-probs and the forward-only loss on the single-turn batch, for profiling")
     ap.add_argument("--lmhead-vocab", type=int, default=0,
                     help="with --lmhead-tokens: a smaller vocabulary, only for small profiling captures")
     ap.add_argument("--prompts", type=int, default=16,
@@ -519,6 +521,38 @@ def tokens_only(args):
                       "frac": 8 * b.N / ms / 1e6 / peak}), flush=True)
 
 
+def logprobs_only(args):
+    """Token log-probs and the forward-only loss alone on the single-turn batch
+    (32,768 x 151,936): --warmup untimed calls, then --steps timed ones of
+    each; prints one JSON line."""
+    from paper_2608_01804_gb300 import build
+    build.build()
+    from paper_2608_01804_gb300 import leap as L
+    from paper_2608_01804_gb300.step import GrpoStep
+    device = torch.device("cuda", 0)
+    batch, logits, ids, old = make_inputs(0, device)
+    step = GrpoStep(batch, V, device, gamma=1.0, tau=(0, batch.G), use_gate_in=False)
+    step.advantages()
+    N = logits.shape[0]
+    live = int((step.w != 0).sum().item())
+    logp = torch.empty(N, dtype=torch.float32, device=device)
+    lse = torch.empty(N, dtype=torch.float32, device=device)
+    ws = L.loss_workspace(N, V, device)
+    lp = lambda: L.leap_token_logprobs(logits, ids, V=V, logp=logp, lse=lse)
+    fwd = lambda: L.leap_grpo_loss_fwd(logits, ids, old, step.adv, step.w, V=V, loss=step.loss, lse=lse,
+                                       want_dlogits=False, want_outputs=False, workspace=ws)
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        lp()
+        fwd()
+    ms_lp = _timed_launches(lp, args.steps, stream)
+    ms_f = _timed_launches(fwd, args.steps, stream)
+    peak, _ = measured_peaks()
+    b_lp, b_f = 2 * V * N + 12 * N, 2 * V * live + 16 * N
+    print(json.dumps({"logprobs_ms": ms_lp, "logprobs_frac": b_lp / ms_lp / 1e6 / peak,
+                      "fwd_ms": ms_f, "fwd_frac": b_f / ms_f / 1e6 / peak}), flush=True)
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -532,6 +566,9 @@ def main():
         return
     if args.tokens_only:
         tokens_only(args)
+        return
+    if args.logprobs_only:
+        logprobs_only(args)
         return
     rank, world, local = dist_env()
     torch.cuda.set_device(local)
