@@ -367,8 +367,7 @@ leap_status_t leap_gemm_bf16_tn_f32(const uint16_t* A, int64_t lda, const uint16
 
 /* Bytes of workspace leap_fused_lmhead_logprobs needs for the gradients in
  * `grads` (0: forward only).  Either gradient adds one 8,192-token chunk of
- * bf16 dlogits (8,192 x V); LEAP_LMHEAD_DHIDDEN adds a transposed copy of W
- * (H x V bf16). */
+ * bf16 dlogits (8,192 x V). */
 size_t leap_fused_lmhead_workspace_size(int64_t N, int32_t H, int32_t V, int32_t grads);
 
 /*

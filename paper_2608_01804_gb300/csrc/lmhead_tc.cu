@@ -10,7 +10,8 @@
 //                partials of the token log-probs;
 //   EPI_DLOGITS  recomputed logits tile -> dlogits = coef (1[v = y] -
 //                softmax) in bf16, into a transient token-chunk buffer;
-//   EPI_STORE    the accumulator as bf16 (dhidden = dlogits . (W^T)^T);
+//   EPI_STORE    the accumulator as bf16 (dhidden = dlogits . W, W read
+//                MN-major in place);
 //   EPI_ACC_F32  the accumulator added into (or stored to) an fp32 matrix:
 //                the weight gradient dW = dlogits^T . hidden, summed over
 //                token chunks, with both operands read MN-major.
@@ -418,22 +419,6 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
 }
 
-// W [V x H] -> WT [H x ldv] through 32 x 32 shared-memory tiles.
-__global__ void __launch_bounds__(256) transpose_bf16_kernel(const uint16_t* __restrict__ W, uint16_t* __restrict__ WT,
-                                                             int32_t V, int32_t H, int64_t ldv) {
-    __shared__ uint16_t tile[32][33];
-    const int64_t v0 = (int64_t)blockIdx.x * 32, h0 = (int64_t)blockIdx.y * 32;
-    for (int r = threadIdx.y; r < 32; r += 8) {
-        const int64_t v = v0 + r, h = h0 + threadIdx.x;
-        if (v < V && h < H) tile[r][threadIdx.x] = W[v * H + h];
-    }
-    __syncthreads();
-    for (int r = threadIdx.y; r < 32; r += 8) {
-        const int64_t h = h0 + r, v = v0 + threadIdx.x;
-        if (h < H && v < V) WT[h * ldv + v] = tile[threadIdx.x][r];
-    }
-}
-
 // Per row: merge the (max, sum) partials, then the clipped surrogate (Eq. 3)
 // and the per-row coefficients of the backward.
 __global__ void __launch_bounds__(256) lmhead_combine_kernel(RowArgs a, const float2* part, const float* zy,
@@ -532,7 +517,6 @@ struct LmheadWorkspace {
     float* rowK;
     float* rowcoef;
     void* loss_ws;
-    uint16_t* WT;
     uint16_t* DL;
     int64_t chunk;
     size_t bytes;
@@ -556,7 +540,6 @@ LmheadWorkspace lmhead_layout(void* base, int64_t N, int32_t H, int32_t V, bool 
     w.rowcoef = reinterpret_cast<float*>(take(N * sizeof(float)));
     w.loss_ws = take(loss_workspace_bytes(N));
     w.chunk = std::min<int64_t>(N, DLOGITS_CHUNK_ROWS);
-    if (with_dhidden) w.WT = reinterpret_cast<uint16_t*>(take((size_t)H * ldv * 2));
     if (with_dhidden || with_dW) w.DL = reinterpret_cast<uint16_t*>(take((size_t)w.chunk * ldv * 2));
     w.bytes = off;
     return w;
@@ -702,16 +685,11 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
     }
     if ((dhidden || dW) && N > 0) {
         // Backward through token chunks of transient bf16 dlogits:
-        //   dhidden_chunk = DL . W      (K = V; DL and a transposed copy of W, both K-major)
+        //   dhidden_chunk = DL . W      (K = V; DL K-major, W read in place MN-major)
         //   dW += DL^T . hidden_chunk   (K = chunk tokens; DL and hidden read MN-major)
         const int64_t ldv = ((int64_t)V + 7) & ~int64_t(7);
-        CUtensorMap tWT;
-        if (dhidden) {
-            dim3 tgrid((unsigned)((V + 31) / 32), (unsigned)((H + 31) / 32));
-            transpose_bf16_kernel<<<tgrid, dim3(32, 8), 0, s>>>(W, L.WT, V, H, ldv);
-            if ((e = cudaGetLastError()) != cudaSuccess) return LEAP_ERR_CUDA;
-            if (!make_tmap(&tWT, L.WT, (uint64_t)V, (uint64_t)H, (uint64_t)ldv * 2, BN)) return LEAP_ERR_CUDA;
-        }
+        CUtensorMap tWt;
+        if (dhidden && !make_tmap_mn(&tWt, W, (uint64_t)H, (uint64_t)V, (uint64_t)H * 2)) return LEAP_ERR_CUDA;
         for (int64_t c0 = 0; c0 < N; c0 += L.chunk) {
             const int64_t cr = std::min<int64_t>(L.chunk, N - c0);
             CUtensorMap tHc;
@@ -740,7 +718,7 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
                 g2.ldo = H;
                 g2.group_m = LEAP_ST_GROUP_M;
                 g2.status = status;
-                if (launch_gemm<EPI_STORE>(tDL, tWT, g2, s) != cudaSuccess) return LEAP_ERR_CUDA;
+                if (launch_gemm<EPI_STORE, false, true>(tDL, tWt, g2, s) != cudaSuccess) return LEAP_ERR_CUDA;
             }
             if (dW) {
                 CUtensorMap tDLt, tHt;
