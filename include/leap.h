@@ -4,7 +4,9 @@
  * arXiv 2608.01804): rank-based tournament advantages gated by
  * Difficulty-Conditioned Pruning, per-turn discounted token advantages, token
  * log-probs over a large vocabulary, and the clipped GRPO surrogate with its
- * dlogits backward.
+ * dlogits backward; and, on the tensor cores (tcgen05), the same loss
+ * straight from the hidden states through the lm-head with its gradients
+ * with respect to the hidden states and the lm-head weight.
  *
  * Conventions for every entry point
  * ---------------------------------
@@ -27,10 +29,11 @@
  *  - bf16 tensors are passed as uint16_t bit patterns.  Row-major matrices
  *    have a leading dimension `ld` (elements); bf16 matrices need a 16-byte
  *    aligned base and ld % 8 == 0.
- *  - No kernel waits on another launch.  The fused loss kernel waits on its
- *    own asynchronous copies and on the other CTAs of its cluster through
- *    mbarriers; every such wait is bounded and, if it ever gave up, the
- *    kernel would set LEAP_DEV_TIMEOUT and finish instead of hanging.
+ *  - No kernel waits on another launch.  The single-read fused loss kernel
+ *    waits on its own asynchronous copies and on the other CTAs of its
+ *    cluster, the tensor-core GEMM on its own TMA loads, MMAs and epilogue,
+ *    all through mbarriers; every such wait is bounded and, if it ever gave
+ *    up, the kernel would set LEAP_DEV_TIMEOUT and finish instead of hanging.
  */
 #ifndef LEAP_H_
 #define LEAP_H_
