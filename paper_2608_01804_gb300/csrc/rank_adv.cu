@@ -252,35 +252,66 @@ __global__ void __launch_bounds__(256, (J <= 2 ? LEAP_RANK_MINB : 1)) rank_adv_k
                 // Without NaN the order is total, so each rollout gets one
                 // 96-bit key that orders exactly as the comparator:
                 // (r, speedup, -tokens) for a pass, 0 for a failure (failures
-                // tie whatever their speedup and tokens).  Strict comparisons
-                // never count a rollout against itself.
-                unsigned long long khi[J];
-                unsigned klo[J];
+                // tie whatever their speedup and tokens).  Peers in other
+                // tiers are counted from the tier histogram; the keys of a
+                // tier are gathered into consecutive slots of the warp's
+                // shared memory, so each passing rollout compares itself only
+                // with its own tier (strict comparisons skip itself).
+                if constexpr (J <= 8) {
+                    __shared__ int4 tkeys[8][32 * J];
+                    unsigned long long khi[J];
+                    unsigned klo[J];
 #pragma unroll
-                for (int j = 0; j < J; ++j) {
-                    const unsigned b = __float_as_uint(sp[j] + 0.f);   // -0 -> +0, equal as floats
-                    const unsigned o = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
-                    khi[j] = r[j] > 0 ? (((unsigned long long)r[j] << 32) | o) : 0ull;
-                    klo[j] = r[j] > 0 ? ~((unsigned)tk[j] ^ 0x80000000u) : 0u;
-                }
+                    for (int j = 0; j < J; ++j) {
+                        const unsigned b = __float_as_uint(sp[j] + 0.f);   // -0 -> +0, equal as floats
+                        const unsigned o = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+                        khi[j] = r[j] > 0 ? (((unsigned long long)r[j] << 32) | o) : 0ull;
+                        klo[j] = r[j] > 0 ? ~((unsigned)tk[j] ^ 0x80000000u) : 0u;
+                    }
+                    const unsigned lt = (1u << lane) - 1u;
+                    int lo[J], cnt[J], pos[J];
 #pragma unroll
-                for (int sidx = 0; sidx < J; ++sidx) {
-                    const int npeer = min(32, G - 32 * sidx);  // uniform across the warp
-                    if (npeer <= 0) break;
-                    __syncwarp();
-                    lkeys[wib][lane] = make_int4((int)(unsigned)khi[sidx], (int)(unsigned)(khi[sidx] >> 32),
-                                                 (int)klo[sidx], 0);
-                    __syncwarp();
-#pragma unroll(J >= 16 ? 1 : 4)
-                    for (int l = 0; l < npeer; ++l) {
-                        const int4 kj = lkeys[wib][l];
-                        const unsigned long long hj = ((unsigned long long)(unsigned)kj.y << 32) | (unsigned)kj.x;
-                        const unsigned lj = (unsigned)kj.z;
+                    for (int j = 0; j < J; ++j) lo[j] = cnt[j] = pos[j] = 0;
+                    int below = 0;
+                    for (int b = 0; b <= M; ++b) {   // tiers in order: slots below_b .. below_b + c_b
+                        int pre = 0;
 #pragma unroll
-                        for (int q = 0; q < J; ++q) {
-                            nw[q] += (khi[q] > hj) || (khi[q] == hj && klo[q] > lj);
-                            nb[q] += (hj > khi[q]) || (hj == khi[q] && lj > klo[q]);
+                        for (int j = 0; j < J; ++j) {
+                            const bool in = valid[j] && r[j] == b;
+                            const unsigned bal = __ballot_sync(0xffffffffu, in);
+                            if (in) {
+                                pos[j] = below + pre + __popc(bal & lt);
+                                lo[j] = below;
+                            }
+                            pre += __popc(bal);
                         }
+#pragma unroll
+                        for (int j = 0; j < J; ++j)
+                            if (valid[j] && r[j] == b) cnt[j] = pre;
+                        below += pre;
+                    }
+                    __syncwarp();
+#pragma unroll
+                    for (int j = 0; j < J; ++j)
+                        if (valid[j] && r[j] > 0)
+                            tkeys[wib][pos[j]] = make_int4((int)(unsigned)khi[j], (int)(unsigned)(khi[j] >> 32),
+                                                           (int)klo[j], 0);
+                    __syncwarp();
+#pragma unroll
+                    for (int j = 0; j < J; ++j) {
+                        int win = 0, loss = 0;
+                        if (valid[j] && r[j] > 0) {
+                            for (int p = lo[j]; p < lo[j] + cnt[j]; ++p) {
+                                const int4 kj = tkeys[wib][p];
+                                const unsigned long long hj =
+                                    ((unsigned long long)(unsigned)kj.y << 32) | (unsigned)kj.x;
+                                const unsigned lj = (unsigned)kj.z;
+                                win += (khi[j] > hj) || (khi[j] == hj && klo[j] > lj);
+                                loss += (hj > khi[j]) || (hj == khi[j] && lj > klo[j]);
+                            }
+                        }
+                        nw[j] = lo[j] + win;                       // every lower tier, then wins in the tier
+                        nb[j] = (below - lo[j] - cnt[j]) + loss;   // every higher tier, then losses
                     }
                 }
             } else {
