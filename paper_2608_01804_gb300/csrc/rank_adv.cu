@@ -77,8 +77,9 @@ __device__ __forceinline__ void group_reward(const RankArgs& a, int G, int M, co
 }
 
 // Training-observability counters of one group (Table 5, Sec. 4.2), added to
-// the warp's row of shared-memory counters by lane 0.
-template <int J>
+// the warp's row of shared-memory counters by lane 0.  MB: a bound on M known
+// at compile time (passes at turns above it cannot occur).
+template <int J, int MB = kMaxM>
 __device__ __forceinline__ void group_stats(long long* cnt, int G, bool gate, const bool (&valid)[J],
                                             const bool (&bad)[J], const int (&pt0)[J], const int (&T)[J],
                                             const float (&Av)[J], int lane) {
@@ -94,12 +95,9 @@ __device__ __forceinline__ void group_stats(long long* cnt, int G, bool gate, co
         first += __popc(__ballot_sync(0xffffffffu, ok && pt == 1));
         later += __popc(__ballot_sync(0xffffffffu, ok && gate && pt >= 2));
         failed_on += __popc(__ballot_sync(0xffffffffu, ok && gate && pt != 1));
-        int tsum = valid[j] ? T[j] : 0;
+        turns += __reduce_add_sync(0xffffffffu, valid[j] ? T[j] : 0);
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) tsum += __shfl_xor_sync(0xffffffffu, tsum, o);
-        turns += tsum;
-#pragma unroll
-        for (int m = 1; m < kMaxM; ++m)
+        for (int m = 1; m < MB; ++m)
             by_turn[m] += __popc(__ballot_sync(0xffffffffu, ok && gate && pt == m + 1));
     }
     if (lane == 0) {
@@ -486,7 +484,7 @@ __global__ void __launch_bounds__(256, LEAP_RANK_PAIR_MINB) rank_pair_kernel(Ran
         }
         if (lane == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
 
-        if (a.stats) group_stats<J>(sst[wib], G, gate, valid, bad, pt0, T, Av, lane);
+        if (a.stats) group_stats<J, M>(sst[wib], G, gate, valid, bad, pt0, T, Av, lane);
     }
     if (a.stats) flush_stats(a, sst);
 }
