@@ -68,7 +68,7 @@ struct RowArgs {
     float* ws_rho;
     uint8_t* ws_flag;
     unsigned int* status;
-    int32_t next_stride;  // fused two-pass kernel: rows between a CTA and the one after it on its SM (0 = none)
+    int32_t next_stride;  // fused two-pass kernel: rows between a CTA's successive rows (its grid size)
 };
 
 // Workspace carve-up of leap_grpo_loss_fwd.

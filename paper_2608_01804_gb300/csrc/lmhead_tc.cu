@@ -36,20 +36,12 @@ namespace {
 
 constexpr int BM = 128;   // tokens per tile (tensor-memory lanes)
 constexpr int BN = 256;   // columns per tile (accumulator columns)
-#ifndef LEAP_TC_BK
-#define LEAP_TC_BK 64
-#endif
-#ifndef LEAP_TC_STAGES
-#define LEAP_TC_STAGES (LEAP_TC_BK == 64 ? 4 : 8)
-#endif
-constexpr int BK = LEAP_TC_BK;  // K per stage: one 128-byte (64) or 64-byte (32) swizzle row of bf16
-constexpr int STAGES = LEAP_TC_STAGES;
-static_assert(BK == 64 || BK == 32, "K-major tiles use the 128- or 64-byte swizzle");
-// K-major tiles: rows of BK bf16 (BK * 2 bytes, the swizzle span), 8-row
-// swizzle atoms KROW_ATOM bytes apart; descriptor swizzle code 2 = 128-byte,
-// 4 = 64-byte.
+constexpr int BK = 64;      // K per stage: one 128-byte swizzle row of bf16
+constexpr int STAGES = 4;   // 4 x 48 KB; 3 stages measured 9 % slower, K = 32 stages (64-byte swizzle) slower still
+// K-major tiles: rows of BK bf16 (128 bytes, the swizzle span), 8-row swizzle
+// atoms KROW_ATOM bytes apart; descriptor swizzle code 2 = 128-byte.
 constexpr uint32_t KROW_ATOM = 8 * BK * 2;
-constexpr uint64_t KSWZ_CODE = (BK == 64) ? 2 : 4;
+constexpr uint64_t KSWZ_CODE = 2;
 constexpr uint32_t A_TILE = BM * BK * 2;
 constexpr uint32_t B_TILE = BN * BK * 2;
 constexpr uint32_t STAGE_BYTES = A_TILE + B_TILE;
@@ -57,15 +49,11 @@ constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
 constexpr int GEMM_THREADS = 192;       // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr size_t GEMM_DYN_SMEM = (size_t)STAGES * STAGE_BYTES + 1024;
 constexpr int LSE_TILES_PER_UNIT = 8;   // 2,048 vocabulary columns per LSE work unit
-#ifndef LEAP_LSE_GROUP_M
-#define LEAP_LSE_GROUP_M 16  // forward: the 152 CTAs in flight cover 16 hidden tiles x ~10 vocabulary units
-#endif
-#ifndef LEAP_DL_GROUP_M
-#define LEAP_DL_GROUP_M 16  // dlogits chunk: 16 token tiles x ~10 vocabulary tiles in flight
-#endif
-#ifndef LEAP_ST_GROUP_M
-#define LEAP_ST_GROUP_M 8   // dhidden: 8 token tiles x 20 hidden tiles (the whole N) in flight
-#endif
+// Token tiles per group of the grouped tile order (measured; see the tile
+// order note at unit_coords):
+constexpr int kLseGroupM = 16;  // forward: the 152 CTAs in flight cover 16 hidden tiles x ~10 vocabulary units
+constexpr int kDlGroupM = 16;   // dlogits chunk: 16 token tiles x ~10 vocabulary tiles in flight
+constexpr int kStGroupM = 8;    // dhidden: 8 token tiles x 20 hidden tiles (the whole N) in flight
 constexpr int64_t DLOGITS_CHUNK_ROWS = 8192;
 
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1),
@@ -152,7 +140,7 @@ __device__ __forceinline__ void tma_load_2d(uint32_t smem_dst, const CUtensorMap
 }
 
 // Shared-memory matrix descriptor of a K-major tile written by TMA with the
-// 128-byte (64-byte) swizzle: rows of BK * 2 bytes, 8-row groups KROW_ATOM
+// 128-byte swizzle: rows of BK * 2 = 128 bytes, 8-row groups KROW_ATOM = 1024
 // bytes apart.  Fields: start address >> 4 (bits 0-13), leading byte offset
 // >> 4 (16-29, unused for this layout), stride byte offset >> 4 (32-45),
 // descriptor version 1 (bit 46), swizzle mode (bits 61-63).
@@ -479,8 +467,7 @@ bool make_tmap_box(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t o
 // A K-major operand: `inner` = K contiguous, boxes of BK x box_outer rows.
 bool make_tmap(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
                uint32_t box_outer) {
-    return make_tmap_box(tm, base, inner, outer, row_bytes, BK, box_outer,
-                         BK == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B);
+    return make_tmap_box(tm, base, inner, outer, row_bytes, BK, box_outer, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 // An MN-major operand: `inner` = M (or N) contiguous, boxes of 64 x BK rows (128-byte swizzle).
 bool make_tmap_mn(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes) {
@@ -570,7 +557,7 @@ extern "C" leap_status_t leap_gemm_bf16_nt(const uint16_t* A, int64_t lda, const
     g.tiles_per_unit = 1;
     g.out = C;
     g.ldo = ldc;
-    g.group_m = LEAP_ST_GROUP_M;
+    g.group_m = kStGroupM;
     g.status = nullptr;
     const cudaError_t e = launch_gemm<EPI_STORE>(ta, tb, g, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? LEAP_OK : LEAP_ERR_CUDA;
@@ -664,7 +651,7 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
         g.N = V;
         g.K = H;
         g.tiles_per_unit = LSE_TILES_PER_UNIT;
-        g.group_m = LEAP_LSE_GROUP_M;
+        g.group_m = kLseGroupM;
         g.part = L.part;
         g.zy = L.zy;
         g.ids = ids;
@@ -704,7 +691,7 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
             g1.rowK = L.rowK + c0;
             g1.rowcoef = L.rowcoef + c0;
             g1.c1 = c1;
-            g1.group_m = LEAP_DL_GROUP_M;
+            g1.group_m = kDlGroupM;
             g1.status = status;
             if (launch_gemm<EPI_DLOGITS>(tHc, tW, g1, s) != cudaSuccess) return LEAP_ERR_CUDA;
             if (dhidden) {
@@ -716,7 +703,7 @@ extern "C" leap_status_t leap_fused_lmhead_logprobs(const leap_loss_params_t* p,
                 g2.K = V;
                 g2.out = dhidden + c0 * H;
                 g2.ldo = H;
-                g2.group_m = LEAP_ST_GROUP_M;
+                g2.group_m = kStGroupM;
                 g2.status = status;
                 if (launch_gemm<EPI_STORE, false, true>(tDL, tWt, g2, s) != cudaSuccess) return LEAP_ERR_CUDA;
             }

@@ -153,14 +153,12 @@ __device__ __forceinline__ void flush_stats(const RankArgs& a, long long (*sst)[
     }
 }
 
-#ifndef LEAP_RANK_MINB
-#define LEAP_RANK_MINB 4
-#endif
-#ifndef LEAP_RANK_PAIR_MINB
-#define LEAP_RANK_PAIR_MINB 6
-#endif
+// Blocks of 256 threads per SM the register budget is cut for (measured: 4
+// for the generic kernel with J <= 2, 6 for the pair kernel).
+constexpr int kRankMinBlocks = 4;
+constexpr int kPairMinBlocks = 6;
 template <int J, bool LEXI>  // rollouts per lane: G <= 32 * J; tie-broken comparator
-__global__ void __launch_bounds__(256, (J <= 2 ? LEAP_RANK_MINB : 1)) rank_adv_kernel(RankArgs a) {
+__global__ void __launch_bounds__(256, (J <= 2 ? kRankMinBlocks : 1)) rank_adv_kernel(RankArgs a) {
     const int lane = threadIdx.x & 31;
     const int wib = threadIdx.x >> 5;
     const int G = a.G, M = a.M;
@@ -392,7 +390,7 @@ __global__ void __launch_bounds__(256, (J <= 2 ? LEAP_RANK_MINB : 1)) rank_adv_k
 // pair with one vector store (the turn advantages as M float2), and the tier
 // walk and the discount loops unroll.
 template <int MC>
-__global__ void __launch_bounds__(256, LEAP_RANK_PAIR_MINB) rank_pair_kernel(RankArgs a) {
+__global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs a) {
     constexpr int J = 2, M = MC;
     const int lane = threadIdx.x & 31;
     const int wib = threadIdx.x >> 5;
@@ -489,15 +487,10 @@ __global__ void __launch_bounds__(256, LEAP_RANK_PAIR_MINB) rank_pair_kernel(Ran
     if (a.stats) flush_stats(a, sst);
 }
 
-#ifndef LEAP_RANK_BLOCKS_PER_SM
-#define LEAP_RANK_BLOCKS_PER_SM 0
-#endif
 template <int J>
 cudaError_t launch_rank_j(const RankArgs& a, cudaStream_t s) {
     const int warps = 8;
     int64_t blocks = ((int64_t)a.num_groups + warps - 1) / warps;
-    if (LEAP_RANK_BLOCKS_PER_SM > 0)
-        blocks = std::min<int64_t>(blocks, (int64_t)device_sm_count() * LEAP_RANK_BLOCKS_PER_SM);
     // With counters, fewer blocks loop over the groups: one atomic set per block.
     if (a.stats) blocks = std::min<int64_t>(blocks, (int64_t)device_sm_count() * 16);
     if (a.cmp == 1) rank_adv_kernel<J, true><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
@@ -575,10 +568,7 @@ __device__ __forceinline__ float recip_count(double x) {
 // of log2 S), then every lane walks forward through the (non-decreasing)
 // offsets as its tokens advance, reloading a segment's fields only when it
 // enters a new segment.
-#ifndef LEAP_SCATTER_ITERS
-#define LEAP_SCATTER_ITERS 8
-#endif
-constexpr int kScatterIters = LEAP_SCATTER_ITERS;
+constexpr int kScatterIters = 8;   // 256 tokens per warp chunk (16 and 4 measured no better)
 
 __global__ void __launch_bounds__(256) scatter_kernel(SegArgs a) {
     const int64_t nv = a.totals_in[0];
