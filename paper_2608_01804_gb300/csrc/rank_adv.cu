@@ -530,6 +530,57 @@ __global__ void segment_count_kernel(SegArgs a) {
     if (t < (int)a.T_eff[i]) atomicAdd(&a.L_out[i], hi - lo);
 }
 
+// The whole count in one launch when the per-rollout counters fit in shared
+// memory: one block zeroes them there, adds every segment with shared-memory
+// atomics, then writes L and the two totals (block barriers instead of three
+// dependent launches).
+constexpr int kCountThreads = 1024;
+constexpr int kCountSmemRollouts = 12000;   // int32 counters within the 48 KB of static shared memory
+
+__global__ void __launch_bounds__(kCountThreads) counts_one_block_kernel(SegArgs a) {
+    __shared__ int32_t sL[kCountSmemRollouts];
+    __shared__ long long st[2][kCountThreads / 32];
+    const int n = a.n_rollouts;
+    for (int i = threadIdx.x; i < n; i += kCountThreads) sL[i] = 0;
+    __syncthreads();
+    for (int64_t s = threadIdx.x; s < a.num_segs; s += kCountThreads) {
+        int32_t lo, hi, i, t;
+        if (!segment_ok(a, s, lo, hi, i, t)) {
+            flag_status(a.status, 4u);
+            continue;
+        }
+        if (t >= 0 && hi > lo && t < (int)a.T_eff[i]) atomicAdd(&sL[i], hi - lo);
+    }
+    __syncthreads();
+    long long tok = 0, roll = 0;
+    for (int i = threadIdx.x; i < n; i += kCountThreads) {
+        const int32_t l = sL[i];
+        a.L_out[i] = l;
+        tok += l;
+        roll += (l > 0);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        tok += __shfl_xor_sync(0xffffffffu, tok, o);
+        roll += __shfl_xor_sync(0xffffffffu, roll, o);
+    }
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        st[0][w] = tok;
+        st[1][w] = roll;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        long long a0 = 0, a1 = 0;
+        for (int k = 0; k < kCountThreads / 32; ++k) {
+            a0 += st[0][k];
+            a1 += st[1][k];
+        }
+        a.totals_out[0] = a0;
+        a.totals_out[1] = a1;
+    }
+}
+
 __global__ void totals_kernel(const int32_t* L, int32_t n, int64_t* totals) {
     long long tok = 0, roll = 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
@@ -677,6 +728,10 @@ cudaError_t launch_rank_advantages(const RankArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_token_counts(const SegArgs& a, cudaStream_t s) {
+    if (a.n_rollouts <= kCountSmemRollouts) {
+        counts_one_block_kernel<<<1, kCountThreads, 0, s>>>(a);
+        return cudaGetLastError();
+    }
     const int sms = device_sm_count();
     const int64_t zb = std::min<int64_t>(((int64_t)a.n_rollouts + 255) / 256, (int64_t)sms * 4);
     zero_counts_kernel<<<(unsigned)std::max<int64_t>(zb, 1), 256, 0, s>>>(a.L_out, a.n_rollouts, a.totals_out);

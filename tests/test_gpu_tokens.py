@@ -37,6 +37,22 @@ def test_counts_and_scatter(maker, agg):
     assert abs(w.astype(np.float64).sum() - 1.0) < 1e-5
 
 
+def test_counts_past_the_one_block_limit():
+    """More rollouts than the one-block count keeps in shared memory (12,000):
+    the three-launch count path, against the oracle."""
+    b = synth.single_turn_batch(seed=5, num_prompts=1600)      # 12,800 rollouts, 3.3 M tokens
+    assert b.n > 12000
+    orc = oracle_rank(b, gamma=0.9)
+    ta32 = orc["turn_adv"].reshape(-1).astype(np.float32)
+    T_eff = orc["T_eff"].reshape(-1)
+    Lc, tot, adv, w = _gpu_tokens(b, ta32, T_eff, O.AGG_SEQ_MEAN_TOKEN_MEAN)
+    L_o, nv, rv, adv_o, w_o = oracle_tokens(b, ta32.astype(np.float64), T_eff, O.AGG_SEQ_MEAN_TOKEN_MEAN)
+    np.testing.assert_array_equal(Lc, L_o)
+    assert tuple(tot) == (nv, rv)
+    np.testing.assert_array_equal(adv, adv_o.astype(np.float32))
+    np.testing.assert_array_equal(w, w_o.astype(np.float32))
+
+
 def test_dcp_pruned_turns_have_zero_weight():
     b = synth.tiny_batch()
     orc = oracle_rank(b, gamma=0.9)
