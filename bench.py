@@ -704,7 +704,7 @@ def main():
                            "vocab": V, "logits_dtype": "bf16", "l2": "inputs larger than L2 (9.96 GB of logits "
                            "read and 9.96 GB of dlogits written per step)", "parallelism": "dp%d" % world},
                 "roofline": roofline, "rows": rows, "cpu_baseline": cpu, "e2e": e2e,
-                "gpu_launches": K * GrpoStep.LAUNCHES_PER_RUN, "clocks": clk}
+                "gpu_launches": K * step.launches_per_run(), "clocks": clk}
         print(json.dumps(line), flush=True)
     if pg is not None:
         torch.distributed.destroy_process_group()

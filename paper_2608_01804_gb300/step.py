@@ -128,5 +128,10 @@ class GrpoStep:
             self._stage_key = key
         return self._stage
 
-    # Kernel launches one run() makes (rank 1, counts 3, scatter 1, loss 1 + reduce 2).
-    LAUNCHES_PER_RUN = 8
+    # libleap counts tokens in one launch up to this many rollouts, three above it.
+    ONE_BLOCK_COUNT_ROLLOUTS = 12000
+
+    def launches_per_run(self):
+        """Kernel launches one run() makes: rank 1, counts 1 (or 3), scatter 1, loss 1 + reduce 2."""
+        counts = 1 if self.b.n <= self.ONE_BLOCK_COUNT_ROLLOUTS else 3
+        return 1 + counts + 1 + 1 + 2
