@@ -40,7 +40,7 @@ WORKLOAD = ("single-turn GRPO: 16 prompts x G=8 x 256 token slots = 32,768 rows 
 # dram bytes (read + write) of one fused_loss_kernel launch on this workload: an ncu capture of the
 # kernel built from sources with this SHA-256 on a 4,096-row slice, scaled to the full launch by
 # algorithmic bytes (traffic grows in proportion to them); null once the sources change.
-KNOWN_TRAFFIC = {"src_sha256": "c66c6c032dc37bc79225c17159a74835ef3dfd6c115e4335560a4575c6624f20", "bytes_per_launch": 16319810859}
+KNOWN_TRAFFIC = {"src_sha256": "485457ae5bfd97e4b93d539a63292f777878268f78af4bab4630090ffd84ec94", "bytes_per_launch": 16305801239}
 KERNEL_SOURCES = ("paper_2608_01804_gb300/csrc/logprob_loss.cu", "paper_2608_01804_gb300/csrc/leap_common.cuh",
                   "paper_2608_01804_gb300/csrc/loss_math.cuh")
 
@@ -643,7 +643,7 @@ def main():
               "frac_of_nominal_7900_gbs": achieved / 7900.0}
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "launch_spread": spread,
-                "traffic": traffic, "kernel": "fused_loss_l2_kernel<1024,4> persistent (+2 reduce launches in the timing)",
+                "traffic": traffic, "kernel": "fused_loss_l2_kernel<1024,4,6> persistent (+2 reduce launches in the timing)",
                 "algorithmic_bytes_per_launch": alg_bytes, "launch_ms": loss_ms, "peak_source": peak_kind}
 
     # End to end through the same public calls, inputs copied from pinned host memory every step.

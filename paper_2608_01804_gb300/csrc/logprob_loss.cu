@@ -395,7 +395,8 @@ __global__ void __launch_bounds__(T + 32, MINB) fused_loss_kernel(RowArgs a, int
 // ---------------------------------------------------------------------------
 // Measured settings (the alternatives are in the kernel's profile summary):
 constexpr int kL2Threads = 1024;           // one CTA per SM (512 x 2 and 256 x 4 overflow L2)
-constexpr int kL2U = 4;                    // 16-byte vectors in flight per thread and pass
+constexpr int kL2U1 = 4;                   // 16-byte vectors in flight per thread, pass 1 (2: 0.850, 8: 0.791)
+constexpr int kL2U2 = 6;                   // and pass 2 (2: 0.824, 4: 0.874, 5-8: 0.882-0.883, 10 spills)
 constexpr int64_t kPfChunk = 32768;        // bytes per bulk L2 prefetch request
 constexpr int64_t kNextBytes = 65536;      // head of the next row prefetched during pass 2
 // Warp-wide: bulk L2 prefetch of the first min(cap, row) bytes of a logits row.
@@ -415,7 +416,7 @@ __device__ __forceinline__ void prefetch_next_row(const RowArgs& a, int64_t row,
 }
 
 // One row of the fused two-pass forward + backward, by the whole CTA.
-template <int T, int U>
+template <int T, int U1, int U2>
 __device__ __forceinline__ void l2_row(const RowArgs& a, const int64_t row, float2* wpart, float* bc) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int V = a.V;
@@ -448,10 +449,10 @@ __device__ __forceinline__ void l2_row(const RowArgs& a, const int64_t row, floa
     if (warp == 0) prefetch_row_l2(zr, V, (int64_t)1 << 40, keep, lane);
     const float c1 = a.inv_temp * kLog2e;
     float m = -INFINITY, s = 0.f;
-    for (int64_t v0 = t; v0 < V8; v0 += (int64_t)T * U) {
-        uint4 x[U];
+    for (int64_t v0 = t; v0 < V8; v0 += (int64_t)T * U1) {
+        uint4 x[U1];
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
+        for (int u = 0; u < U1; ++u) {
             const int64_t vi = v0 + (int64_t)u * T;
             x[u] = (vi < V8) ? ld_stream_hint(zrow + vi, keep) : neg_inf4();
             if (tailn && vi == V8 - 1) mask_tail(x[u], tailn);
@@ -484,23 +485,23 @@ __device__ __forceinline__ void l2_row(const RowArgs& a, const int64_t row, floa
     const uint64_t drop = l2_policy_evict_first();
     const int64_t yv = id >> 3;
     const int ylane = id & 7;
-    for (int64_t v0 = t; v0 < V8; v0 += (int64_t)T * U) {
+    for (int64_t v0 = t; v0 < V8; v0 += (int64_t)T * U2) {
         if (coef == 0.f) {
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
+            for (int u = 0; u < U2; ++u) {
                 const int64_t vi = v0 + (int64_t)u * T;
                 if (vi < V8) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
             }
             continue;
         }
-        uint4 x[U];
+        uint4 x[U2];
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
+        for (int u = 0; u < U2; ++u) {
             const int64_t vi = v0 + (int64_t)u * T;
             x[u] = (vi < V8) ? ld_stream_hint(zrow + vi, drop) : neg_inf4();
         }
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
+        for (int u = 0; u < U2; ++u) {
             const int64_t vi = v0 + (int64_t)u * T;
             if (vi < V8) store_vec(drow, vi, dlogit8(x[u], c1, K, coef, vi == yv ? ylane : -1), V8, tailn);
         }
@@ -510,11 +511,11 @@ __device__ __forceinline__ void l2_row(const RowArgs& a, const int64_t row, floa
 // One persistent CTA per SM walks rows blockIdx.x, + gridDim.x, ... with no
 // CTA launch between rows (the round-robin spreads masked and live rows
 // evenly; one CTA per row measured 0.845 of the copy peak against 0.871).
-template <int T, int U>
+template <int T, int U1, int U2>
 __global__ void __launch_bounds__(T, 1) fused_loss_l2_kernel(RowArgs a) {
     __shared__ float2 wpart[T / 32];
     __shared__ float bc[2];
-    for (int64_t row = blockIdx.x; row < a.N; row += gridDim.x) l2_row<T, U>(a, row, wpart, bc);
+    for (int64_t row = blockIdx.x; row < a.N; row += gridDim.x) l2_row<T, U1, U2>(a, row, wpart, bc);
 }
 
 // ---------------------------------------------------------------------------
@@ -781,7 +782,7 @@ cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s
         RowArgs b = a;
         const int64_t grid = std::min<int64_t>(a.N, (int64_t)device_sm_count());
         b.next_stride = (int32_t)grid;   // exactly the CTA's next row
-        fused_loss_l2_kernel<kL2Threads, kL2U><<<(unsigned)grid, kL2Threads, 0, s>>>(b);
+        fused_loss_l2_kernel<kL2Threads, kL2U1, kL2U2><<<(unsigned)grid, kL2Threads, 0, s>>>(b);
         return cudaGetLastError();
     }
     const int64_t V8 = ((int64_t)a.V + 7) >> 3;
