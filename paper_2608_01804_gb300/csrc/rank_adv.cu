@@ -416,13 +416,14 @@ __global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs
         }
         bool valid[J] = {own, own}, bad[J];
         int pt0[J], r[J];
-        int n_fail = 0;
+        int fails = 0;
 #pragma unroll
         for (int j = 0; j < J; ++j) {
             bool fail1;
             decode_outcome(pt[j], T[j], M, valid[j], bad[j], fail1, pt0[j]);
-            n_fail += __popc(__ballot_sync(0xffffffffu, fail1));
+            fails += fail1;
         }
+        const int n_fail = __reduce_add_sync(0xffffffffu, fails);
         const bool gate = a.gate_in ? (a.gate_in[group] != 0) : (a.tau_min <= n_fail && n_fail <= a.tau_max);
 #pragma unroll
         for (int j = 0; j < J; ++j) {
@@ -430,25 +431,43 @@ __global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs
             if (bad[j]) flag_status(a.status, 2u);
         }
 
-        // Eq. 5 for the paper's comparator: the ordered tier walk.
-        int nw[J] = {0, 0}, eq[J] = {0, 0}, below = 0;
+        // Eq. 5 for the paper's comparator: the tier histogram as 8-bit
+        // counters packed four to a word (a group holds at most 64), summed
+        // over the warp with one reduction per word; the byte-wise prefix
+        // (multiplication by 0x01010101) gives each tier its count of peers
+        // in lower tiers.
+        constexpr int W = (M + 4) / 4;   // words for the M + 1 tiers
+        unsigned hist[W], pre[W];
 #pragma unroll
-        for (int b = 0; b <= M; ++b) {
-            const int c = __popc(__ballot_sync(0xffffffffu, own && r[0] == b)) +
-                          __popc(__ballot_sync(0xffffffffu, own && r[1] == b));
+        for (int w = 0; w < W; ++w) {
+            unsigned mine = 0;
 #pragma unroll
-            for (int j = 0; j < J; ++j) {
-                if (r[j] == b) {
-                    nw[j] = below;
-                    eq[j] = c;
-                }
-            }
-            below += c;
+            for (int j = 0; j < J; ++j)
+                if (own && (r[j] >> 2) == w) mine += 1u << (8 * (r[j] & 3));
+            hist[w] = __reduce_add_sync(0xffffffffu, mine);
         }
-        int nb[J], d[J];
+        unsigned carry = 0;   // peers in the tiers of earlier words
+#pragma unroll
+        for (int w = 0; w < W; ++w) {
+            pre[w] = hist[w] * 0x01010101u + carry * 0x01010101u;   // inclusive prefix per byte
+            carry = pre[w] >> 24;
+        }
+        const int below = (int)carry;   // == G
+        int nw[J], nb[J], d[J];
 #pragma unroll
         for (int j = 0; j < J; ++j) {
-            nb[j] = below - nw[j] - eq[j];
+            const int w = r[j] >> 2, k = r[j] & 3;
+            unsigned hw = hist[0], pw = pre[0];
+#pragma unroll
+            for (int q = 1; q < W; ++q)
+                if (w == q) {
+                    hw = hist[q];
+                    pw = pre[q];
+                }
+            const int eq = (int)((hw >> (8 * k)) & 0xffu);
+            const int incl = (int)((pw >> (8 * k)) & 0xffu);   // peers in tiers <= r (this one included)
+            nw[j] = incl - eq;
+            nb[j] = below - incl;
             d[j] = nw[j] - nb[j];
         }
         const int dd = __reduce_add_sync(0xffffffffu, own ? d[0] * d[0] + d[1] * d[1] : 0);
