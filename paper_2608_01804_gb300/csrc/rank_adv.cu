@@ -245,24 +245,22 @@ __global__ void __launch_bounds__(256, (J <= 2 ? kRankMinBlocks : 1)) rank_adv_k
                 keyed = !__any_sync(0xffffffffu, nan_key);
             }
             if (keyed) {
-                // Without NaN the order is total, so each rollout gets one
-                // 96-bit key that orders exactly as the comparator:
-                // (r, speedup, -tokens) for a pass, 0 for a failure (failures
-                // tie whatever their speedup and tokens).  Peers in other
-                // tiers are counted from the tier histogram; the keys of a
-                // tier are gathered into consecutive slots of the warp's
-                // shared memory, so each passing rollout compares itself only
-                // with its own tier (strict comparisons skip itself).
+                // Without NaN the order within a tier is total: each passing
+                // rollout gets one 64-bit key (speedup, -tokens) that orders
+                // exactly as the comparator's tie-breaks.  Peers in other
+                // tiers are counted from the tier histogram (failures tie
+                // whatever their speedup and tokens); the keys of a tier are
+                // gathered into consecutive slots of the warp's shared memory,
+                // so each passing rollout compares itself only with its own
+                // tier (strict comparisons skip itself).
                 if constexpr (J <= 8) {
-                    __shared__ int4 tkeys[8][32 * J];
-                    unsigned long long khi[J];
-                    unsigned klo[J];
+                    __shared__ unsigned long long tkeys[8][32 * J];
+                    unsigned long long key[J];
 #pragma unroll
                     for (int j = 0; j < J; ++j) {
                         const unsigned b = __float_as_uint(sp[j] + 0.f);   // -0 -> +0, equal as floats
                         const unsigned o = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
-                        khi[j] = r[j] > 0 ? (((unsigned long long)r[j] << 32) | o) : 0ull;
-                        klo[j] = r[j] > 0 ? ~((unsigned)tk[j] ^ 0x80000000u) : 0u;
+                        key[j] = ((unsigned long long)o << 32) | ~((unsigned)tk[j] ^ 0x80000000u);
                     }
                     const unsigned lt = (1u << lane) - 1u;
                     int lo[J], cnt[J], pos[J];
@@ -289,21 +287,16 @@ __global__ void __launch_bounds__(256, (J <= 2 ? kRankMinBlocks : 1)) rank_adv_k
                     __syncwarp();
 #pragma unroll
                     for (int j = 0; j < J; ++j)
-                        if (valid[j] && r[j] > 0)
-                            tkeys[wib][pos[j]] = make_int4((int)(unsigned)khi[j], (int)(unsigned)(khi[j] >> 32),
-                                                           (int)klo[j], 0);
+                        if (valid[j] && r[j] > 0) tkeys[wib][pos[j]] = key[j];
                     __syncwarp();
 #pragma unroll
                     for (int j = 0; j < J; ++j) {
                         int win = 0, loss = 0;
                         if (valid[j] && r[j] > 0) {
                             for (int p = lo[j]; p < lo[j] + cnt[j]; ++p) {
-                                const int4 kj = tkeys[wib][p];
-                                const unsigned long long hj =
-                                    ((unsigned long long)(unsigned)kj.y << 32) | (unsigned)kj.x;
-                                const unsigned lj = (unsigned)kj.z;
-                                win += (khi[j] > hj) || (khi[j] == hj && klo[j] > lj);
-                                loss += (hj > khi[j]) || (hj == khi[j] && lj > klo[j]);
+                                const unsigned long long kp = tkeys[wib][p];
+                                win += key[j] > kp;
+                                loss += kp > key[j];
                             }
                         }
                         nw[j] = lo[j] + win;                       // every lower tier, then wins in the tier
