@@ -369,8 +369,8 @@ leap_status_t leap_gemm_bf16_tn_f32(const uint16_t* A, int64_t lda, const uint16
 #define LEAP_LMHEAD_DW 2
 
 /* Bytes of workspace leap_fused_lmhead_logprobs needs for the gradients in
- * `grads` (0: forward only).  Either gradient adds one 8,192-token chunk of
- * bf16 dlogits (8,192 x V). */
+ * `grads` (0: forward only).  Either gradient adds one chunk of bf16 dlogits
+ * (min(N, 16,384) x V: 5 GB at V = 151,936). */
 size_t leap_fused_lmhead_workspace_size(int64_t N, int32_t H, int32_t V, int32_t grads);
 
 /*
@@ -379,7 +379,7 @@ size_t leap_fused_lmhead_workspace_size(int64_t N, int32_t H, int32_t V, int32_t
  * then exactly leap_grpo_loss_fwd's outputs (loss, logp, lse, ell, stats;
  * ids, old_logp, adv, w as there; params->flags may hold
  * LEAP_LOSS_ACCUMULATE).  Gradients of the loss (chain rule through z,
- * from bf16 dlogits recomputed for 8,192-token chunks):
+ * from bf16 dlogits recomputed for 16,384-token chunks):
  *   dhidden  bf16 [N x H], nullable: d loss / d hidden = dlogits . W;
  *   dW       fp32 [V x H], nullable, 16-byte aligned: d loss / d W =
  *            dlogits^T . hidden, summed over all N tokens in fp32 (chunk by

@@ -54,7 +54,7 @@ constexpr int LSE_TILES_PER_UNIT = 8;   // 2,048 vocabulary columns per LSE work
 constexpr int kLseGroupM = 16;  // forward: the 152 CTAs in flight cover 16 hidden tiles x ~10 vocabulary units
 constexpr int kDlGroupM = 16;   // dlogits chunk: 16 token tiles x ~10 vocabulary tiles in flight
 constexpr int kStGroupM = 8;    // dhidden: 8 token tiles x 20 hidden tiles (the whole N) in flight
-constexpr int64_t DLOGITS_CHUNK_ROWS = 8192;
+constexpr int64_t DLOGITS_CHUNK_ROWS = 16384;
 
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1),
 // A and B bf16 (bits 7-9 = 1, 10-12 = 1), A / B major-ness at bits 15 / 16
