@@ -52,7 +52,7 @@ constexpr int LSE_TILES_PER_UNIT = 8;   // 2,048 vocabulary columns per LSE work
 // Token tiles per group of the grouped tile order (measured; see the tile
 // order note at unit_coords):
 constexpr int kLseGroupM = 16;  // forward: the 152 CTAs in flight cover 16 hidden tiles x ~10 vocabulary units
-constexpr int kDlGroupM = 16;   // dlogits chunk: 16 token tiles x ~10 vocabulary tiles in flight
+constexpr int kDlGroupM = 32;   // dlogits chunk: 32 token tiles x ~5 vocabulary tiles in flight
 constexpr int kStGroupM = 8;    // dhidden: 8 token tiles x 20 hidden tiles (the whole N) in flight
 constexpr int64_t DLOGITS_CHUNK_ROWS = 16384;
 
