@@ -375,8 +375,41 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
     del dl, ws
     torch.cuda.synchronize()
 
-    # a8: fused lm-head (tcgen05), 65,536 tokens x H = 5,120 x V = 151,936.
+    # The whole pass (a1-a7) on the small workload (4 prompts x 8 x 2 turns x
+    # 256 = 16,384 rows, V = 1,024; 32 MB of logits, resident in L2), where the
+    # host's launches cost more than the kernels: 100 back-to-back steps
+    # launched kernel by kernel, then as replays of one CUDA graph.
     from paper_2608_01804_gb300.step import GrpoStep
+    tb = synth.tiny_batch()
+    Vt = 1024
+    zt = synth.logits(tb.N, Vt, 2.0, 700, device)
+    it = synth.token_ids(tb.N, Vt, 701, device)
+    ot = torch_logp(zt, it) + synth.normal(tb.N, 0.05, 702, device)
+    st_t = GrpoStep(tb, Vt, device, gamma=0.9, tau=(0, tb.G))
+    dl_t = torch.empty_like(zt)
+    graph = st_t.capture(zt, it, ot, dl_t)
+
+    def back_to_back(fn, k=100):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        a.record(stream)
+        for _ in range(k):
+            fn()
+        b.record(stream)
+        b.synchronize()
+        return a.elapsed_time(b) / k
+
+    eager_ms = back_to_back(lambda: st_t.run(zt, it, ot, dl_t))
+    graph_ms = back_to_back(graph.replay)
+    nv_t = valid_tokens(tb)
+    rows["step_tiny_16384xV1024_eager_vs_graph"] = {
+        "eager_ms": eager_ms, "graph_ms": graph_ms, "launches_per_step": st_t.launches_per_run(),
+        "eager_valid_tokens_per_s": nv_t / (eager_ms / 1e3), "graph_valid_tokens_per_s": nv_t / (graph_ms / 1e3),
+        "note": "100 back-to-back steps, host launch cost included, logits resident in L2"}
+    del graph, st_t, zt, dl_t
+    torch.cuda.synchronize()
+
+    # a8: fused lm-head (tcgen05), 65,536 tokens x H = 5,120 x V = 151,936.
     lb = synth.lmhead_batch()
     N8, H = lb.N, 5120
     hidden = synth.normal((N8, H), 1.0, 500, device, dtype=torch.bfloat16)

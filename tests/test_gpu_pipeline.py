@@ -160,3 +160,40 @@ def test_streamed_step_equals_resident_step():
     assert loss_str.item() == expect.item()
     # The whole-batch loss differs from the chunked one only by the fp32 sum over chunks.
     assert abs(loss_str.item() - loss_res.item()) <= 4 * 2.0 ** -24 * float(step.w.abs().sum().item()) * 2.0
+
+
+def test_graph_replay_equals_eager_step():
+    """GrpoStep.capture: one CUDA-graph replay of the whole pass gives the
+    eager run's loss, dlogits, advantages and weights bit for bit, and a
+    replay after the inputs are refilled in place matches an eager run on the
+    new inputs (the graph reads the buffers, it does not freeze them)."""
+    from paper_2608_01804_gb300.step import GrpoStep
+    L = leap()
+    b = synth.tiny_batch()
+    V = 1024
+    z = synth.logits(b.N, V, 2.0, 220, "cuda")
+    ids = synth.token_ids(b.N, V, 221, "cuda")
+    old = torch_logp(z, ids, V) + synth.normal(b.N, 0.05, 222, "cuda")
+    eager = GrpoStep(b, V, "cuda", gamma=0.9, tau=(0, 8))
+    dl_e = torch.empty_like(z)
+    loss_e = eager.run(z, ids, old, dl_e).clone()
+    graphed = GrpoStep(b, V, "cuda", gamma=0.9, tau=(0, 8))
+    dl_g = torch.full_like(z, 7)
+    g = graphed.capture(z, ids, old, dl_g)
+    dl_g.fill_(7)
+    graphed.loss.fill_(123.0)
+    g.replay()
+    torch.cuda.synchronize()
+    assert L.leap_get_device_status() == 0
+    assert graphed.loss.item() == loss_e.item()
+    assert torch.equal(dl_g, dl_e)
+    assert torch.equal(graphed.adv, eager.adv) and torch.equal(graphed.w, eager.w)
+    # New logits and old log-probs in the same buffers.
+    z2 = synth.logits(b.N, V, 2.0, 223, "cuda")
+    z.copy_(z2)
+    old.copy_(torch_logp(z2, ids, V) + synth.normal(b.N, 0.05, 224, "cuda"))
+    g.replay()
+    loss_e2 = eager.run(z, ids, old, dl_e).clone()
+    torch.cuda.synchronize()
+    assert graphed.loss.item() == loss_e2.item() and graphed.loss.item() != loss_e.item()
+    assert torch.equal(dl_g, dl_e)
