@@ -8,8 +8,7 @@ CUDA library (``paper_2608_01804_gb300``) and imports nothing from it.
 Every function follows the paper (LEAP: Lean Environment-Feedback via Adaptive
 Pruning, arXiv 2608.01804) in its own order and notation, in float64, with
 numpy used only for whole-array primitives (max, exp, log, sum, matmul).
-Where the paper is silent the function states the reading it takes; the same
-readings are listed in the design doc.
+Where the paper is silent the function states the reading it takes.
 
 Pins (what checks this oracle against something other than itself) live in
 ``tests/test_oracle_*.py``.  No function here is "parity unpinned".
