@@ -72,6 +72,9 @@ def parse_args():
                     help="run only the token counts + scatter on the packed multi-turn batch, for profiling captures")
     ap.add_argument("--logprobs-only", action="store_true",
                     help="run only the log-probs and the forward-only loss on the single-turn batch, for profiling")
+    ap.add_argument("--short-rows", action="store_true",
+                    help="run only the fused loss fwd + bwd on short vocabularies (1,024-32,768), default and "
+                         "single-read kernel")
     ap.add_argument("--lmhead-vocab", type=int, default=0,
                     help="with --lmhead-tokens: a smaller vocabulary, only for small profiling captures")
     ap.add_argument("--prompts", type=int, default=16,
@@ -554,6 +557,42 @@ def tokens_only(args):
                       "frac": 8 * b.N / ms / 1e6 / peak}), flush=True)
 
 
+def short_rows(args):
+    """The fused loss forward + backward (with its two reduction launches) on
+    short vocabularies, through the default entry point and with
+    LEAP_LOSS_SINGLE_READ: --warmup untimed calls, then --steps timed ones of
+    each, each after an L2 flush; one JSON line per (V, rows).  Rows of
+    V <= 8,192 take the single-read kernel either way."""
+    from paper_2608_01804_gb300 import build
+    build.build()
+    from paper_2608_01804_gb300 import leap as L
+    from paper_2608_01804_gb300 import synth
+    device = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream()
+    flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    peak, _ = measured_peaks()
+    for Vs, N in [(1024, 16384), (1024, 262144), (4096, 65536), (8192, 32768), (16384, 16384), (32768, 8192)]:
+        z = synth.logits(N, Vs, 2.0, 1, device)
+        ids = synth.token_ids(N, Vs, 2, device)
+        old = torch.full((N,), -7.0, device=device)
+        adv = synth.normal(N, 1.0, 3, device)
+        w = torch.full((N,), 1.0 / N, device=device)
+        dl = torch.empty_like(z)
+        ws = L.loss_workspace(N, Vs, device)
+        loss = torch.zeros(1, device=device)
+        line = {"V": Vs, "rows": N, "algorithmic_bytes": 4 * Vs * N}
+        for name, sr in (("default", False), ("single_read", True)):
+            fn = lambda sr=sr: L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=Vs, loss=loss, dlogits=dl,
+                                                    want_outputs=False, workspace=ws, single_read=sr)
+            for _ in range(max(1, args.warmup)):
+                fn()
+            ms = _timed_launches(fn, args.steps, stream, lambda: flush_buf.fill_(1), lead_cycles=LEAD_CYCLES)
+            line[name + "_us"] = ms * 1e3
+            line[name + "_frac"] = 4 * Vs * N / ms / 1e6 / peak
+        print(json.dumps(line), flush=True)
+        del z, dl, ws
+
+
 def logprobs_only(args):
     """Token log-probs and the forward-only loss alone on the single-turn batch
     (32,768 x 151,936): --warmup untimed calls, then --steps timed ones of
@@ -602,6 +641,9 @@ def main():
         return
     if args.logprobs_only:
         logprobs_only(args)
+        return
+    if args.short_rows:
+        short_rows(args)
         return
     rank, world, local = dist_env()
     torch.cuda.set_device(local)
