@@ -206,8 +206,8 @@ def rank_advantages(pass_turn, num_turns, M, tau_min, tau_max, gamma,
 
 
 def rank_stats(out, pass_turn, M):
-    """Training-observability counters (Table 5, Sec. 4.2) from rank_advantages'
-    results: activated groups, per-rollout and per-group recovery, passes by
+    """Training-observability counters (Table 5, Sec. 4.3; turns per pass:
+    Table 2, Sec. 4.2) from rank_advantages' results: activated groups, per-rollout and per-group recovery, passes by
     turn, total effective turns and passed samples (turns per pass)."""
     gate = np.asarray(out["gate"]).astype(bool)
     T_eff = np.asarray(out["T_eff"])
@@ -218,12 +218,48 @@ def rank_stats(out, pass_turn, M):
     later = on & (pt >= 2)                              # recovered after a first-turn failure
     failed_first_on = on & (pt != 1)
     passes_by_turn = [int(np.sum(first)) if m == 1 else int(np.sum(later & (pt == m))) for m in range(1, 9)]
+    composition, groups_by_bucket = rank_composition(out, M)
     return dict(groups=int(gate.size), gated_groups=int(gate.sum()), rollouts=int(pt.size),
                 nonzero_adv_rollouts=int(np.count_nonzero(np.abs(out["A"]) > 1e-9)),
                 first_turn_passes=int(first.sum()), later_passes=int(later.sum()),
                 groups_with_recovery=int(np.sum(np.any(later, axis=1))),
                 failed_first_turn_in_gated=int(failed_first_on.sum()),
-                total_turns=int(T_eff.sum()), passes_by_turn=passes_by_turn)
+                total_turns=int(T_eff.sum()), passes_by_turn=passes_by_turn,
+                composition=composition.tolist(), groups_by_bucket=groups_by_bucket.tolist())
+
+
+PASS_BUCKETS = 10
+
+
+def rank_composition(out, M, buckets=PASS_BUCKETS):
+    """Rollout composition of Fig. 4 (Sec. 4.5) from rank_advantages' results.
+
+    Readings (the figure itself is not in the text):
+      * a group's "observed pass rate" is its first-turn pass rate
+        p = (G - N_fail) / G, with N_fail of Eq. 1 (the quantity the DCP gate
+        sees, defined alike for LEAP and for multi-turn GRPO);
+      * the buckets are ten equal-width bins of p, b = min(9, floor(10 p)),
+        taken in exact integer arithmetic as min(9, (10 (G - N_fail)) // G);
+      * outcome type from the effective tier r: immediate pass (r = M, a pass
+        at turn 1), debug-assisted pass (0 < r < M, a later pass of an expanded
+        group), failure (r = 0; later passes of a gated-off group never ran);
+      * only rollouts with a nonzero advantage count (|A| > 1e-9 in fp64), split
+        by the sign of A (0: positive, 1: negative).
+    Returns (composition int64 [buckets, 3, 2], groups per bucket int64 [buckets]).
+    """
+    r = np.asarray(out["r"], dtype=np.int64)
+    A = np.asarray(out["A"], dtype=np.float64)
+    n_fail = np.asarray(out["n_fail"], dtype=np.int64)
+    num_groups, G = r.shape
+    bucket = np.minimum(buckets - 1, (buckets * (G - n_fail)) // G)
+    groups_by_bucket = np.bincount(bucket, minlength=buckets).astype(np.int64)
+    kind = np.where(r == M, 0, np.where(r > 0, 1, 2))
+    sign = np.where(A > 0, 0, 1)
+    counted = np.abs(A) > 1e-9
+    b_full = np.broadcast_to(bucket[:, None], r.shape)
+    flat = (b_full * 3 + kind) * 2 + sign
+    composition = np.bincount(flat[counted], minlength=buckets * 6).astype(np.int64)
+    return composition.reshape(buckets, 3, 2), groups_by_bucket
 
 
 # ---------------------------------------------------------------------------

@@ -79,6 +79,30 @@ def test_loss_clip_branches_hand_built():
     np.testing.assert_allclose(out["g"], [0.0, 0.0, -1.1, -1.5, 3.0], rtol=1e-12)
 
 
+def test_loss_asymmetric_clip_hand_built():
+    """Asymmetric clip range eps_low = 0.1, eps_high = 0.28 (Eq. 3 with the two
+    edges 0.9 and 1.28), values by hand; tokens 0 and 1 sit where swapping the
+    two epsilons, or using 0.2 for both, would change their branch."""
+    z = np.zeros((4, 8))          # uniform: logp = -log 8
+    ids = np.zeros(4, dtype=int)
+    lp = -np.log(8.0)
+    rho = np.array([1.25, 0.85, 1.35, 0.95])
+    adv = np.array([1.0, -2.0, 0.5, -1.0])
+    old = lp - np.log(rho)
+    w = np.array([1.0, 0.5, 2.0, 1.0])
+    out = O.grpo_loss_rows(z, ids, old, adv, w, eps_low=0.1, eps_high=0.28)
+    # A>0, rho=1.25 <= 1.28: unclipped, ell = -1.25 ; A<0, rho=0.85 < 0.9: clipped,
+    # ell = -min(-1.7, -1.8) = 1.8 ; A>0, rho=1.35 > 1.28: ell = -1.28*0.5 = -0.64 ;
+    # A<0, rho=0.95 >= 0.9: unclipped, ell = 0.95.
+    np.testing.assert_allclose(out["ell"], [-1.25, 1.8, -0.64, 0.95], rtol=1e-12)
+    np.testing.assert_array_equal(out["active"], [True, False, False, True])
+    np.testing.assert_allclose(out["g"], [-1.25, 0.0, 0.0, 0.95], rtol=1e-12)
+    np.testing.assert_allclose(out["loss"], -1.25 + 0.9 - 1.28 + 0.95, rtol=1e-12)
+    # The symmetric 0.2 range decides tokens 0 and 1 the other way.
+    sym = O.grpo_loss_rows(z, ids, old, adv, w, eps_low=0.2, eps_high=0.2)
+    np.testing.assert_array_equal(sym["active"], [False, True, False, True])
+
+
 def _fd_check(z, ids, old, adv, w, inv_temp, grad_scale, eps_low=0.2, eps_high=0.28):
     out = O.grpo_loss_rows(z, ids, old, adv, w, eps_low, eps_high, inv_temp, grad_scale)
     h = 1e-6

@@ -293,3 +293,55 @@ def test_rank_stats_by_hand():
     assert (st["groups_with_recovery"], st["failed_first_turn_in_gated"]) == (1, 3)
     assert st["total_turns"] == 1 + 2 + 3 + 3 + 4
     assert st["passes_by_turn"][:3] == [2, 1, 1]
+
+
+def test_rank_composition_by_hand():
+    """Fig. 4 counts (Sec. 4.5) on four groups of G = 4, M = 3, worked by hand.
+    Group 0, expanded: turn-1 pass x2, turn-2 pass, failure; 2 of 4 passed turn 1
+    (bucket 5); r = 3, 3, 2, 0 so d = 2, 2, -1, -3.  Group 1, not expanded: its
+    turn-2 pass never ran (a failure), one turn-1 pass; 1 of 4 (bucket 2);
+    r = 0, 0, 0, 3 so d = -1, -1, -1, 3.  Group 2: all fail (bucket 0), group 3:
+    all pass at turn 1 (bucket 9); both all-tied, so A = 0 and nothing counts."""
+    pt = np.array([[1, 1, 2, 0], [2, 0, 0, 1], [0, 0, 0, 0], [1, 1, 1, 1]])
+    nt = np.array([[1, 1, 2, 3], [2, 1, 1, 1], [1, 1, 1, 1], [1, 1, 1, 1]])
+    gate = np.array([1, 0, 0, 0])
+    expect = np.zeros((10, 3, 2), dtype=np.int64)
+    expect[5, 0, 0] = 2      # immediate passes, A > 0
+    expect[5, 1, 1] = 1      # debug-assisted pass, A < 0 (beaten by both turn-1 passes)
+    expect[5, 2, 1] = 1      # failure, A < 0
+    expect[2, 0, 0] = 1
+    expect[2, 2, 1] = 3      # includes the truncated turn-2 pass
+    groups = [1, 0, 1, 0, 0, 1, 0, 0, 0, 1]
+    for reward in (O.REWARD_RANK, O.REWARD_STATIC):   # static 1 / 0.5 / 0 gives the same signs here
+        out = O.rank_advantages(pt, nt, 3, 0, 4, 0.9, gate_in=gate, reward=reward, static_c=0.5)
+        comp, gb = O.rank_composition(out, 3)
+        np.testing.assert_array_equal(comp, expect)
+        assert gb.tolist() == groups
+        st = O.rank_stats(out, pt, 3)
+        assert st["composition"] == expect.tolist() and st["groups_by_bucket"] == groups
+        assert int(comp.sum()) == st["nonzero_adv_rollouts"] == 8
+
+
+def test_rank_composition_invariants():
+    """On a random batch: every nonzero-advantage rollout is counted once, every
+    group sits in one bucket, groups whose rollouts all pass turn 1 land in the
+    last bucket and those with none in the first, and with M = 1 there is no
+    debug-assisted pass."""
+    rng = np.random.default_rng(5)
+    for G, M in ((8, 3), (16, 1), (64, 3), (5, 2)):
+        n = 300
+        T = rng.integers(1, M + 1, size=(n, G))
+        pt = np.where(rng.random((n, G)) < 0.5, rng.integers(1, M + 1, size=(n, G)), 0)
+        pt = np.minimum(pt, T)
+        pt[0] = 1
+        pt[1] = 0
+        out = O.rank_advantages(pt, T, M, 2, G - 2, 0.9)
+        comp, gb = O.rank_composition(out, M)
+        st = O.rank_stats(out, pt, M)
+        assert int(comp.sum()) == st["nonzero_adv_rollouts"]
+        assert int(gb.sum()) == n
+        b = np.minimum(9, (10 * (G - out["n_fail"])) // G)
+        assert b[0] == 9 and b[1] == 0
+        np.testing.assert_array_equal(np.bincount(b, minlength=10), gb)
+        if M == 1:
+            assert comp[:, 1, :].sum() == 0
