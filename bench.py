@@ -37,7 +37,7 @@ WORKLOAD = ("single-turn GRPO: 16 prompts x G=8 x 256 token slots = 32,768 rows 
             "rest masked padding), V=151936, bf16 logits N(0,3^2) + 1% spikes of +15, old log-probs = current "
             "+ N(0,0.05^2), clip eps 0.2/0.2, seq-mean-token-mean aggregation")
 
-# dram bytes (read + write) of one fused_loss_kernel launch on this workload: an ncu capture of the
+# dram bytes (read + write) of one fused_loss_l2_kernel launch on this workload: an ncu capture of the
 # kernel built from sources with this SHA-256 on a 4,096-row slice, scaled to the full launch by
 # algorithmic bytes (traffic grows in proportion to them); null once the sources change.
 KNOWN_TRAFFIC = {"src_sha256": "485457ae5bfd97e4b93d539a63292f777878268f78af4bab4630090ffd84ec94", "bytes_per_launch": 16305801239}
@@ -75,11 +75,27 @@ def parse_args():
     ap.add_argument("--short-rows", action="store_true",
                     help="run only the fused loss fwd + bwd on short vocabularies (1,024-32,768), default and "
                          "single-read kernel")
+    ap.add_argument("--short-case", default="",
+                    help="with --short-rows: one case VxROWS (e.g. 1024x131072) instead of the sweep")
+    ap.add_argument("--multiturn", action="store_true",
+                    help="run only the whole pass on the packed multi-turn DCP workload (chunked)")
     ap.add_argument("--lmhead-vocab", type=int, default=0,
                     help="with --lmhead-tokens: a smaller vocabulary, only for small profiling captures")
     ap.add_argument("--prompts", type=int, default=16,
                     help="prompts per rank (16 = the benchmark workload; fewer only for profiling captures)")
     return ap.parse_args()
+
+
+def _cpu_model():
+    """The host CPU's model name (lscpu), for the record beside the oracle's rate."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return None
 
 
 def dist_env():
@@ -212,6 +228,71 @@ def cpu_oracle_rate(batch, logits, ids, old, seconds, block=32):
     return valid / t_total, rows, valid, t_total
 
 
+# ---- the oracle on every host core (a process pool started with spawn) ----
+_SHM = {}
+
+
+def _pool_init(shm_name, shape):
+    """Worker start-up: one thread per worker, attach the shared logits bits."""
+    from multiprocessing import shared_memory
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[k] = "1"
+    shm = shared_memory.SharedMemory(name=shm_name)
+    _SHM["shm"] = shm
+    _SHM["bits"] = np.ndarray(shape, dtype=np.uint16, buffer=shm.buf)
+
+
+def _pool_rows(task):
+    """The oracle's loss forward and dlogits on rows [a, b) (weights w != 0 only are read)."""
+    from oracle import leap_oracle as O
+    a, b, ids, old, adv, w = task
+    live = np.nonzero(w)[0]
+    if len(live) == 0:
+        return 0
+    z = O.bf16_bits_to_f64(_SHM["bits"][a:b][live])
+    O.grpo_loss_rows(z, ids[live], old[live], adv[live], w[live])
+    return len(live)
+
+
+def cpu_oracle_rate_all_cores(batch, logits, ids, old, block=32):
+    """The oracle (as it stands) over the WHOLE batch on every host core: the
+    rank/token steps once, then the loss forward + dlogits of every row in
+    blocks of `block` rows, spread over os.cpu_count() spawned workers that
+    read the bf16 logits from host shared memory.  Returns (valid tokens/s,
+    workers, valid tokens, seconds)."""
+    import multiprocessing as mp
+    from multiprocessing import shared_memory
+    from oracle import leap_oracle as O
+    G, M = batch.G, batch.M
+    N, Vr = logits.shape
+    workers = os.cpu_count() or 1
+    shm = shared_memory.SharedMemory(create=True, size=N * Vr * 2)
+    try:
+        bits = np.ndarray((N, Vr), dtype=np.uint16, buffer=shm.buf)
+        for a0 in range(0, N, 4096):
+            b0 = min(N, a0 + 4096)
+            bits[a0:b0] = logits[a0:b0].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+        ids_h = ids.cpu().numpy().astype(np.int64)
+        old_h = old.cpu().numpy().astype(np.float64)
+        ctx = mp.get_context("spawn")
+        with ctx.Pool(workers, initializer=_pool_init, initargs=(shm.name, (N, Vr))) as pool:
+            pool.map(_pool_rows, [(0, 0, ids_h[:0], old_h[:0], old_h[:0], old_h[:0])] * workers)   # start-up
+            t0 = time.perf_counter()
+            orc = O.rank_advantages(batch.pass_turn.reshape(-1, G), batch.num_turns.reshape(-1, G), M, 0, G, 1.0)
+            ta, te = orc["turn_adv"].reshape(-1), orc["T_eff"].reshape(-1)
+            Lc, nv, rv = O.rollout_token_counts(batch.seg_offsets, batch.seg_rollout, batch.seg_turn, te)
+            adv, w = O.token_advantages(batch.N, batch.seg_offsets, batch.seg_rollout, batch.seg_turn, ta, te, M, 0,
+                                        Lc, nv, rv)
+            tasks = [(a, min(N, a + block), ids_h[a:a + block], old_h[a:a + block], adv[a:a + block], w[a:a + block])
+                     for a in range(0, N, block)]
+            valid = sum(pool.imap_unordered(_pool_rows, tasks, chunksize=1))
+            secs = time.perf_counter() - t0
+        return valid / secs, workers, valid, secs
+    finally:
+        shm.close()
+        shm.unlink()
+
+
 def reference_arm(args):
     """The oracle (fp64 CPU) as the reference implementation, timed per step on
     a bounded sample of the same workload; rank 0 only."""
@@ -286,6 +367,56 @@ def _timed_launches(fn, reps, stream, flush=None, lead_cycles=0):
     return total / reps
 
 
+MT_CHUNK = 65536   # rows per logits chunk of the multi-turn stream
+
+
+def multiturn_step(device, peak, steps=3, warmup=1):
+    """The whole pass on the packed multi-turn DCP workload (32 prompts x G = 16,
+    up to 3 turns, prompts and feedback masked, ~1.49 M rows, V = 151,936)
+    through GrpoStep.run_chunked: rank -> counts -> scatter over the whole
+    stream, then the fused loss over 65,536-row chunks with loss accumulation.
+    The stream's 452 GB of logits exceed HBM, so one 65,536-row chunk of logits
+    (19.9 GB, N(0, 3^2) + 1% spikes) is drawn once and stands in for every chunk
+    (the ids, old log-probs, advantages and weights are the true per-row ones);
+    dlogits go to one chunk buffer likewise.  Each chunk is larger than L2."""
+    from paper_2608_01804_gb300 import synth
+    from paper_2608_01804_gb300.step import GrpoStep
+    b = synth.multiturn_dcp_batch()
+    N = b.N
+    zbuf = synth.logits(MT_CHUNK, V, 3.0, 300, device, spike_frac=0.01)
+    dlbuf = torch.empty_like(zbuf)
+    ids = synth.token_ids(N, V, 301, device)
+    old = torch.empty(N, dtype=torch.float32, device=device)
+    for a in range(0, N, MT_CHUNK):   # current-policy log-probs of each chunk's rows (input generation)
+        n = min(MT_CHUNK, N - a)
+        old[a:a + n] = torch_logp(zbuf[:n], ids[a:a + n])
+    old += synth.normal(N, 0.05, 302, device)
+    step = GrpoStep(b, V, device, gamma=0.9, tau=(8, 15), use_gate_in=False, chunk_rows=MT_CHUNK)
+    chunks = [(a, zbuf[:min(MT_CHUNK, N - a)], dlbuf[:min(MT_CHUNK, N - a)]) for a in range(0, N, MT_CHUNK)]
+    for _ in range(max(1, warmup)):
+        step.run_chunked(chunks, ids, old)
+    torch.cuda.synchronize()
+    live = int((step.w != 0).sum().item())
+    stream = torch.cuda.current_stream()
+    a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a_ev.record(stream)
+    for _ in range(steps):
+        step.run_chunked(chunks, ids, old)
+    b_ev.record(stream)
+    b_ev.synchronize()
+    ms = a_ev.elapsed_time(b_ev) / steps
+    alg = live * 4 * V + (N - live) * 2 * V + 16 * N
+    gbs = alg / (ms / 1e3) / 1e9
+    out = {"ms_per_step": ms, "rows": N, "valid_tokens": live, "chunks": len(chunks), "algorithmic_bytes": alg,
+           "achieved_gbs": gbs, "frac": gbs / peak, "throughput": live / (ms / 1e3), "unit": "valid tokens/s",
+           "launches_per_step": 1 + (1 if b.n <= GrpoStep.ONE_BLOCK_COUNT_ROLLOUTS else 3) + 1 + 3 * len(chunks),
+           "note": "whole step (rank, counts, scatter, fused loss + reductions per chunk); one 65,536-row "
+                   "logits chunk reused for every chunk"}
+    del zbuf, dlbuf, step
+    torch.cuda.synchronize()
+    return out
+
+
 def measure_rows(device, logits, ids, old, step, peak, reps=5):
     """Each remaining row of the hot path on its own workload, against the HBM
     roofline: rank advantages on 65,536 groups x 64 rollouts (M = 3), token
@@ -351,6 +482,9 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
     ms = _timed_launches(tok, reps * 4, stream, flush, lead_cycles=LEAD_CYCLES)
     rows["token_counts_scatter_multiturn_%d_tokens" % b.N] = entry(8 * b.N, ms, b.N, "tokens/s")
     del adv, w
+
+    # The whole pass on the multi-turn DCP workload (a1-a7 over the chunked stream).
+    rows["multiturn_dcp_step_%d_rows_V151936" % b.N] = multiturn_step(device, peak)
 
     # a5: log-probs (2V bytes per row), and the split forward / backward (a6, a7).
     N = logits.shape[0]
@@ -571,7 +705,10 @@ def short_rows(args):
     stream = torch.cuda.current_stream()
     flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device=device)
     peak, _ = measured_peaks()
-    for Vs, N in [(1024, 16384), (1024, 262144), (4096, 65536), (8192, 32768), (16384, 16384), (32768, 8192)]:
+    cases = [(1024, 16384), (1024, 262144), (4096, 65536), (8192, 32768), (16384, 16384), (32768, 8192)]
+    if args.short_case:
+        cases = [tuple(int(x) for x in args.short_case.split("x"))]
+    for Vs, N in cases:
         z = synth.logits(N, Vs, 2.0, 1, device)
         ids = synth.token_ids(N, Vs, 2, device)
         old = torch.full((N,), -7.0, device=device)
@@ -644,6 +781,14 @@ def main():
         return
     if args.short_rows:
         short_rows(args)
+        return
+    if args.multiturn:
+        from paper_2608_01804_gb300 import build
+        build.build()
+        torch.cuda.set_device(0)
+        peak, _ = measured_peaks()
+        print(json.dumps(multiturn_step(torch.device("cuda", 0), peak, steps=args.steps, warmup=args.warmup)),
+              flush=True)
         return
     rank, world, local = dist_env()
     torch.cuda.set_device(local)
@@ -765,10 +910,16 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rate, n_rows, valid, secs = cpu_oracle_rate(batch, logits, ids, old, args.cpu_seconds)
-        cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
-               "sample": "rank/token oracle on the whole batch + loss fwd and dlogits on the first %d rows "
-                         "(%d valid tokens), %.1f s of CPU time" % (n_rows, valid, secs)}
+        rate1, n_rows, valid1, secs1 = cpu_oracle_rate(batch, logits, ids, old, args.cpu_seconds)
+        rate, workers, valid, secs = cpu_oracle_rate_all_cores(batch, logits, ids, old)
+        cpu = {"value": rate, "unit": UNIT, "cores": workers, "kind": "oracle",
+               "sample": "the whole batch (%d valid tokens): rank/token oracle once, then loss fwd and dlogits of "
+                         "every row in 32-row blocks over %d spawned worker processes, %.1f s wall"
+                         % (valid, workers, secs),
+               "cpu_model": _cpu_model(),
+               "single_thread": {"value": rate1, "cores": 1,
+                                 "sample": "rank/token oracle on the whole batch + loss fwd and dlogits on the first "
+                                           "%d rows (%d valid tokens), %.1f s of CPU time" % (n_rows, valid1, secs1)}}
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,

@@ -97,11 +97,23 @@ typedef enum {
 } leap_reward_t;
 
 /* Training-observability counters of a leap_group_rank_advantages call
- * (Table 5, Sec. 4.2).  Device struct, ACCUMULATED (+=): zero it first.
+ * (activated groups and recovery rates: Table 5, Sec. 4.3; turns per pass:
+ * Table 2, Sec. 4.2).  Device struct, ACCUMULATED (+=): zero it first.
  *   activated-group rate  = gated_groups / groups
  *   per-rollout recovery  = later_passes / failed_first_turn_in_gated
  *   per-group recovery    = groups_with_recovery / gated_groups
  *   turns per pass        = total_turns / (first_turn_passes + later_passes) */
+#define LEAP_PASS_BUCKETS 10
+/* Rollout composition (Fig. 4, Sec. 4.5).  A group's observed pass rate is its
+ * first-turn pass rate p = (G - N_fail) / G (Eq. 1's count, the quantity the
+ * DCP gate sees); it falls in bucket b = min(9, floor(10 p)), computed exactly
+ * as min(9, (10 (G - N_fail)) div G), i.e. ten equal-width buckets with p = 1
+ * in the last.  Each rollout with A != 0 is counted in
+ * composition[b][type][sign]: type 0 = immediate pass (tier r = M, a turn-1
+ * pass), 1 = debug-assisted pass (0 < r < M, a pass at a later turn of an
+ * expanded group), 2 = failure (r = 0, including later passes a gated-off
+ * group never ran); sign 0 = A > 0, 1 = A < 0.  Fig. 4's per-bucket
+ * percentages are composition[b][.][.] over its sum for bucket b. */
 typedef struct {
     int64_t groups, gated_groups;
     int64_t rollouts, nonzero_adv_rollouts;
@@ -111,6 +123,8 @@ typedef struct {
     int64_t failed_first_turn_in_gated; /* rollouts of gated groups that failed turn 1 */
     int64_t total_turns;                /* sum of the effective turn counts */
     int64_t passes_by_turn[8];          /* [m - 1]: passes at turn m (turn 1 from any group) */
+    int64_t composition[LEAP_PASS_BUCKETS][3][2]; /* nonzero-advantage rollouts, see above */
+    int64_t groups_by_bucket[LEAP_PASS_BUCKETS];  /* groups per observed-pass-rate bucket */
 } leap_rank_stats_t;
 
 typedef struct {
@@ -242,8 +256,9 @@ leap_status_t leap_token_logprobs(
  * CTAs that hold it in registers, so it is read from HBM exactly once whatever
  * else is using L2 (supports V <= 262,144).  The default kernel reads a row
  * twice, the second time from L2, which is faster when the loss pass has the
- * GPU's L2 to itself.  Rows of V <= 8,192 take the single-read kernel (one CTA
- * per row) with or without the flag: on such short rows it is 2.5-5x faster. */
+ * GPU's L2 to itself.  Rows of V <= 8,192 take a third kernel with or without
+ * the flag: a group of 1-8 warps holds each row in registers (read once) and
+ * reduces it with warp shuffles. */
 #define LEAP_LOSS_SINGLE_READ 2u
 
 typedef struct {
@@ -399,6 +414,26 @@ leap_status_t leap_fused_lmhead_logprobs(
     void* workspace, size_t ws_bytes,
     leap_loss_stats_t* stats,
     void* stream);
+
+/* ------------------------------------------------------------------------
+ * 6. Self-test of the failure path (library diagnostics; the paper has no
+ *    counterpart).
+ * ------------------------------------------------------------------------ */
+
+/*
+ * Every wait inside a libleap kernel (on its own asynchronous copies, its
+ * tensor-core work or its cluster peers) is bounded: if it ever gave up, the
+ * kernel would set LEAP_DEV_TIMEOUT and return instead of hanging the GPU.
+ * This call exercises that give-up path on purpose: one thread of a tiny
+ * kernel waits, through the same bounded wait, on a barrier that nothing
+ * completes, for limit_ns nanoseconds of GPU wall time (1,000 .. 10^10),
+ * then sets LEAP_DEV_TIMEOUT and returns; leap_get_device_status() then
+ * reports it.  waited_ns (device uint64, nullable) receives the time the wait
+ * took before giving up.  Nothing is in flight when it gives up, so the
+ * context stays usable.  Returns LEAP_ERR_INVALID_ARG for a limit out of
+ * range, LEAP_ERR_CUDA if the launch fails.
+ */
+leap_status_t leap_selftest_bounded_wait(uint64_t limit_ns, uint64_t* waited_ns, void* stream);
 
 #ifdef __cplusplus
 }

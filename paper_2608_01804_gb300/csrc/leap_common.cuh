@@ -183,7 +183,7 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr unsigned int kDevTimeout = 8u;
 template <bool kCluster>
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, unsigned int* status,
-                                                  volatile int* abort_flag) {
+                                                  volatile int* abort_flag, uint64_t limit_ns = kWaitLimitNs) {
     auto poll = [&]() { return kCluster ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity); };
     if (poll()) return true;
     if (*abort_flag) return false;
@@ -193,7 +193,7 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
         for (int i = 0; i < 64; ++i)
             if (poll()) return true;
         if (*abort_flag) return false;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        if (globaltimer_ns() - t0 > limit_ns) {
             *abort_flag = 1;
             flag_status(status, kDevTimeout);
             return false;

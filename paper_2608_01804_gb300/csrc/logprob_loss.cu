@@ -17,6 +17,10 @@
 //                      exchange one (max, sum) pair through distributed
 //                      shared memory: each row is read from HBM exactly once
 //                      whatever else uses L2 (LEAP_LOSS_SINGLE_READ).
+//   short_row_kernel   forward + backward for V <= 8,192: a group of 1-8
+//                      warps holds one row in registers (read once) and
+//                      reduces it with warp shuffles; persistent groups load
+//                      the next row while they write the current one.
 //   split_bwd_kernel   dlogits from a saved lse: 2V read + 2V written.
 //   reduce kernels     fixed-order fp64 sum of the per-row loss terms.
 #include "../../include/leap.h"
@@ -519,6 +523,163 @@ __global__ void __launch_bounds__(T, 1) fused_loss_l2_kernel(RowArgs a) {
 }
 
 // ---------------------------------------------------------------------------
+// Fused forward + backward for short rows (V <= 8,192).  A row group of W
+// warps owns one row at a time; thread t of the group holds vectors
+// t, t + 32W, ... (NV of them) of the row in registers, so the row is read
+// from HBM once.  The (max, sum) reduction is a warp butterfly (every lane
+// ends with the row's value), and for W > 1 one named barrier per live row
+// merges the W warp partials through shared memory (two alternating slots).
+// Row groups are persistent and walk rows g, g + stride, ... with a three-deep
+// pipeline: while row i is reduced and written, the vectors and target logit
+// of row i + 1 are being loaded into registers and row i + kShortAhead has a
+// bulk L2 prefetch in flight (no register cost), so the register loads hit L2
+// and each SM keeps several rows' reads in flight.  Masked rows are not read.
+// ---------------------------------------------------------------------------
+constexpr int kShortThreads = 256;        // 8 warps per CTA
+constexpr int kShortNV = 4;               // 16-byte vectors per thread and row
+constexpr int kShortMinBlocks = 3;        // register budget: 80 per thread, no spills
+constexpr int kShortAhead = 3;            // rows between the L2 prefetch and the row's use
+constexpr bool kShortRegPrefetch = true;  // next row's vectors loaded into registers a row early
+
+template <int W>
+__global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kernel(RowArgs a) {
+    constexpr int NV = kShortNV, TG = 32 * W, GPB = kShortThreads / TG;
+    static_assert(kShortAhead == 3, "the scalar pipeline below holds rows i .. i + 3");
+    __shared__ float2 part[2][kShortThreads / 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int gib = warp / W;                  // row group within the block
+    const int t = (warp % W) * 32 + lane;      // thread within the row group
+    // 32-bit row and vector indices (N < 2^31 is checked on the host; V8 <= 1,024).
+    const int stride = (int)gridDim.x * GPB;
+    const int N = (int)a.N;
+    const int V = a.V;
+    const int V8 = (V + 7) >> 3;
+    const int tailn = V & 7;
+    const float c1 = a.inv_temp * kLog2e;
+    const uint64_t keep = l2_policy_evict_last();
+    const uint64_t drop = l2_policy_evict_first();
+
+    auto is_live = [&](float wr, int idr) { return wr != 0.f && idr >= 0 && idr < V; };
+    auto load_row = [&](int r, int idr, uint4 (&v)[NV], float& z) {
+        const uint16_t* zr = a.logits + (int64_t)r * a.ld;
+        const uint4* zrow = reinterpret_cast<const uint4*>(zr);
+#pragma unroll
+        for (int k = 0; k < NV; ++k) {
+            const int vi = t + k * TG;
+            v[k] = (vi < V8) ? ld_stream_hint(zrow + vi, drop) : neg_inf4();
+        }
+        z = bf16_at(zr + idr);
+    };
+    // One thread of the group asks L2 for the whole row (at most 16 KB).
+    auto prefetch_row = [&](int r) {
+        if (t == 0) bulk_prefetch_l2(a.logits + (int64_t)r * a.ld, (uint32_t)V8 * 16u, keep);
+    };
+    // w and id of the row `k` strides after `r`, or (0, 0) past the end.
+    auto scalars = [&](int r, int k, float& wr, int& idr) {
+        wr = 0.f;
+        idr = 0;
+        if (r < N - k * stride) {   // r + k * stride < N without overflow
+            wr = a.w[r + k * stride];
+            idr = a.ids[r + k * stride];
+        }
+    };
+
+    int row = (int)blockIdx.x * GPB + gib;
+    // Scalars of rows i .. i + 3 (the last pair is loaded one iteration ahead of its use).
+    float w0, w1, w2, w3;
+    int id0, id1, id2, id3;
+    scalars(row, 0, w0, id0);
+    scalars(row, 1, w1, id1);
+    scalars(row, 2, w2, id2);
+    scalars(row, 3, w3, id3);
+    if (is_live(w1, id1)) prefetch_row(row + stride);
+    if (is_live(w2, id2)) prefetch_row(row + 2 * stride);
+    uint4 x[NV];
+    float zy = 0.f;
+    if (kShortRegPrefetch && row < N && is_live(w0, id0)) load_row(row, id0, x, zy);
+    int par = 0;
+
+    for (; row < N; row += stride) {
+        // Row i + 1: its vectors into registers (its lines are in L2 or on the way).
+        uint4 y[NV];
+        float zyn = 0.f;
+        if (kShortRegPrefetch) {
+            if (is_live(w1, id1)) load_row(row + stride, id1, y, zyn);
+        } else if (is_live(w0, id0)) {
+            load_row(row, id0, x, zy);
+        }
+        // Row i + 3: L2 prefetch; row i + 4: its scalars.
+        if (is_live(w3, id3)) prefetch_row(row + 3 * stride);
+        float w4;
+        int id4;
+        scalars(row, 4, w4, id4);
+
+        const bool bad = (w0 != 0.f) && (id0 < 0 || id0 >= V);
+        uint4* drow = reinterpret_cast<uint4*>(a.dlogits + (int64_t)row * a.ld);
+        if (w0 == 0.f || bad) {   // masked row: the same branch in every warp of the group
+#pragma unroll
+            for (int k = 0; k < NV; ++k) {
+                const int vi = t + k * TG;
+                if (vi < V8) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
+            }
+            if (t == 0) {
+                write_masked_outputs(a, row);
+                if (bad) flag_status(a.status, LEAP_DEV_BAD_ID);
+            }
+        } else {
+            const float old = a.old_logp[row], A = a.adv[row];
+            if (tailn) {
+#pragma unroll
+                for (int k = 0; k < NV; ++k)
+                    if (t + k * TG == V8 - 1) mask_tail(x[k], tailn);
+            }
+            float m = tree_max(x);
+            float ssum = (m != -INFINITY) ? tree_exp_sum(x, c1, m * c1) : 0.f;
+            warp_lse_merge(m, ssum, c1);
+            if (W > 1) {
+                if (lane == 0) part[par][warp] = make_float2(m, ssum);
+                named_bar_sync(1 + gib, TG);
+                const float2 p = (lane < W) ? part[par][gib * W + lane] : make_float2(-INFINITY, 0.f);
+                m = p.x;
+                ssum = p.y;
+                warp_lse_merge(m, ssum, c1);
+                par ^= 1;   // live rows alternate slots: a slot is rewritten only after the
+                            // next live row's barrier, which every reader of it has passed
+            }
+            const TokenLoss r = token_loss(a, m, ssum, zy, old, A, w0);
+            const float K = fmaf(m, c1, log2f(ssum));
+            const float coef = a.grad_scale * r.g * a.inv_temp;
+            if (t == 0) write_row_outputs(a, row, r, w0);
+            const int yv = id0 >> 3;
+            const int ylane = id0 & 7;
+#pragma unroll
+            for (int k = 0; k < NV; ++k) {
+                const int vi = t + k * TG;
+                if (vi < V8) {
+                    const uint4 d = (coef == 0.f) ? make_uint4(0, 0, 0, 0)
+                                                  : dlogit8(x[k], c1, K, coef, vi == yv ? ylane : -1);
+                    store_vec(drow, vi, d, V8, tailn);
+                }
+            }
+        }
+        // Shift the pipeline by one row.
+        if (kShortRegPrefetch) {
+#pragma unroll
+            for (int k = 0; k < NV; ++k) x[k] = y[k];
+            zy = zyn;
+        }
+        w0 = w1;
+        id0 = id1;
+        w1 = w2;
+        id1 = id2;
+        w2 = w3;
+        id2 = id3;
+        w3 = w4;
+        id3 = id4;
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Split backward from the saved lse.  Every thread recomputes the row's scalar
 // coefficient from broadcast loads, so no block synchronisation is needed.
 // ---------------------------------------------------------------------------
@@ -659,8 +820,9 @@ struct FusedCfg {
 // register budget for three CTAs per SM (51 resident clusters).
 constexpr int kBigStages = 1;
 constexpr int kBigMinBlocks = 3;
+// Rows of V <= 8,192 never reach this kernel (they take short_row_kernel).
 constexpr FusedCfg kFused[] = {
-    {1, 128, 1, 4}, {1, 256, 4, 3}, {2, 256, 8, 2}, {4, 256, 10, 2}, {8, 256, 10, 2}, {8, 256, 16, 2},
+    {2, 256, 8, 2}, {4, 256, 10, 2}, {8, 256, 10, 2}, {8, 256, 16, 2},
 };
 
 template <int C, int T, int NV, int STAGES, int MINB = 1>
@@ -776,8 +938,43 @@ cudaError_t launch_split_bwd(const RowArgs& a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+// Persistent grid of the short-row kernel: the CTAs that fit at once (cached
+// per device), at most one row group per row.
+template <int W>
+cudaError_t launch_short_rows(const RowArgs& a, cudaStream_t s) {
+    static std::mutex mu;
+    static int cached_dev = -1, cached_resident = 0;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    int resident = 0;   // CTAs resident at once on the whole device
+    {
+        std::lock_guard<std::mutex> lk(mu);
+        if (cached_dev != dev) {
+            int per_sm = 0;
+            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, short_row_kernel<W>, kShortThreads, 0);
+            if (e != cudaSuccess) return e;
+            cached_dev = dev;
+            cached_resident = per_sm * device_sm_count();
+        }
+        resident = cached_resident;
+    }
+    if (resident <= 0) return cudaErrorNotSupported;
+    constexpr int GPB = kShortThreads / (32 * W);
+    const int64_t blocks = std::min<int64_t>((a.N + GPB - 1) / GPB, (int64_t)resident);
+    short_row_kernel<W><<<(unsigned)blocks, kShortThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s) {
     if (a.N == 0) return cudaSuccess;
+    const int64_t V8s = ((int64_t)a.V + 7) >> 3;
+    if (V8s <= (int64_t)8 * 32 * kShortNV) {   // V <= 8,192: the row lives in one row group's registers
+        if (V8s <= 32 * kShortNV) return launch_short_rows<1>(a, s);
+        if (V8s <= 2 * 32 * kShortNV) return launch_short_rows<2>(a, s);
+        if (V8s <= 4 * 32 * kShortNV) return launch_short_rows<4>(a, s);
+        return launch_short_rows<8>(a, s);
+    }
     if (!single_read) {
         RowArgs b = a;
         const int64_t grid = std::min<int64_t>(a.N, (int64_t)device_sm_count());
@@ -789,8 +986,6 @@ cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s
     for (const FusedCfg& c : kFused) {
         const int64_t per = (V8 + c.C - 1) / c.C;
         if (per > (int64_t)c.T * c.NV) continue;
-        if (c.C == 1 && c.T == 128) return launch_fused_cfg<1, 128, 1, 4>(a, s);
-        if (c.C == 1) return launch_fused_cfg<1, 256, 4, 3>(a, s);
         if (c.C == 2) return launch_fused_cfg<2, 256, 8, 2, 2>(a, s);
         if (c.C == 4) return launch_fused_cfg<4, 256, 10, 2, 2>(a, s);
         if (c.NV == 10) return launch_fused_cfg<8, 256, 10, kBigStages, kBigMinBlocks>(a, s);

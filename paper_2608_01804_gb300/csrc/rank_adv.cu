@@ -25,8 +25,13 @@ __device__ __forceinline__ float warp_sum_f(float v) {
     return v;
 }
 
-// Per-warp running counters (lane 0), reduced per block then added atomically.
-constexpr int kNumStats = 9 + kMaxM;
+// Per-warp running counters (lane 0), reduced per block then added atomically;
+// the order of leap_rank_stats_t: 9 scalars, passes by turn, the rollout
+// composition [bucket][type][sign], groups per bucket.
+constexpr int kPassBuckets = 10;
+constexpr int kCompBase = 9 + kMaxM;
+constexpr int kBucketBase = kCompBase + kPassBuckets * 6;
+constexpr int kNumStats = kBucketBase + kPassBuckets;
 
 // Eq. 6 and the advantage of every rollout the lane holds: the tournament
 // reward with the GRPO step, or the static-scalar baseline reward.
@@ -76,17 +81,25 @@ __device__ __forceinline__ void group_reward(const RankArgs& a, int G, int M, co
     }
 }
 
-// Training-observability counters of one group (Table 5, Sec. 4.2), added to
-// the warp's row of shared-memory counters by lane 0.  MB: a bound on M known
-// at compile time (passes at turns above it cannot occur).
+// Training-observability counters of one group (Table 5, Sec. 4.3; Table 2,
+// Sec. 4.2) and its rollout composition (Fig. 4, Sec. 4.5), added to the
+// warp's row of shared-memory counters by lane 0.  MB: a bound on M known at
+// compile time (passes at turns above it cannot occur).  The composition
+// bucket is the group's first-turn pass rate, min(9, 10 (G - N_fail) div G);
+// a rollout with A != 0 counts by type (r = M immediate pass, 0 < r < M
+// debug-assisted pass, r = 0 failure) and by the sign of A.
 template <int J, int MB = kMaxM>
-__device__ __forceinline__ void group_stats(long long* cnt, int G, bool gate, const bool (&valid)[J],
-                                            const bool (&bad)[J], const int (&pt0)[J], const int (&T)[J],
-                                            const float (&Av)[J], int lane) {
+__device__ __forceinline__ void group_stats(long long* cnt, int G, int M, bool gate, int n_fail,
+                                            const bool (&valid)[J], const bool (&bad)[J], const int (&pt0)[J],
+                                            const int (&T)[J], const int (&r)[J], const float (&Av)[J],
+                                            int lane) {
     int nonzero = 0, first = 0, later = 0, failed_on = 0, turns = 0;
     int by_turn[kMaxM];
+    int comp[6];
 #pragma unroll
     for (int m = 0; m < kMaxM; ++m) by_turn[m] = 0;
+#pragma unroll
+    for (int c = 0; c < 6; ++c) comp[c] = 0;
 #pragma unroll
     for (int j = 0; j < J; ++j) {
         const bool ok = valid[j] && !bad[j];
@@ -99,6 +112,11 @@ __device__ __forceinline__ void group_stats(long long* cnt, int G, bool gate, co
 #pragma unroll
         for (int m = 1; m < MB; ++m)
             by_turn[m] += __popc(__ballot_sync(0xffffffffu, ok && gate && pt == m + 1));
+        // Composition category (type * 2 + sign), -1 for A == 0.
+        const int kind = (r[j] == M) ? 0 : ((r[j] > 0) ? 1 : 2);
+        const int cat = (valid[j] && Av[j] != 0.f) ? kind * 2 + (Av[j] < 0.f ? 1 : 0) : -1;
+#pragma unroll
+        for (int c = 0; c < 6; ++c) comp[c] += __popc(__ballot_sync(0xffffffffu, cat == c));
     }
     if (lane == 0) {
         long long* c = cnt;
@@ -114,6 +132,10 @@ __device__ __forceinline__ void group_stats(long long* cnt, int G, bool gate, co
         c[9] += first;
 #pragma unroll
         for (int m = 1; m < kMaxM; ++m) c[9 + m] += by_turn[m];
+        const int bucket = min(kPassBuckets - 1, (kPassBuckets * (G - n_fail)) / G);
+#pragma unroll
+        for (int k = 0; k < 6; ++k) c[kCompBase + bucket * 6 + k] += comp[k];
+        c[kBucketBase + bucket] += 1;
     }
     __syncwarp();
 }
@@ -371,7 +393,7 @@ __global__ void __launch_bounds__(256, (J <= 2 ? kRankMinBlocks : 1)) rank_adv_k
         }
         if (lane == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
 
-        if (a.stats) group_stats<J>(sst[wib], G, gate, valid, bad, pt0, T, Av, lane);
+        if (a.stats) group_stats<J>(sst[wib], G, M, gate, n_fail, valid, bad, pt0, T, r, Av, lane);
     }
 
     if (a.stats) flush_stats(a, sst);
@@ -494,7 +516,7 @@ __global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs
         }
         if (lane == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
 
-        if (a.stats) group_stats<J, M>(sst[wib], G, gate, valid, bad, pt0, T, Av, lane);
+        if (a.stats) group_stats<J, M>(sst[wib], G, M, gate, n_fail, valid, bad, pt0, T, r, Av, lane);
     }
     if (a.stats) flush_stats(a, sst);
 }

@@ -40,6 +40,7 @@ LEAP_LOSS_ACCUMULATE = 1
 LEAP_LOSS_SINGLE_READ = 2
 LEAP_LMHEAD_DHIDDEN = 1
 LEAP_LMHEAD_DW = 2
+LEAP_PASS_BUCKETS = 10
 
 # Every symbol include/leap.h declares.
 EXPORTS = (
@@ -47,7 +48,7 @@ EXPORTS = (
     "leap_group_rank_advantages", "leap_rollout_token_counts", "leap_scatter_turn_advantages",
     "leap_token_logprobs", "leap_grpo_loss_workspace_size", "leap_grpo_loss_fwd", "leap_grpo_loss_bwd",
     "leap_grpo_loss_fwd_noalloc", "leap_gemm_bf16_nt", "leap_gemm_bf16_tn_f32", "leap_fused_lmhead_workspace_size",
-    "leap_fused_lmhead_logprobs",
+    "leap_fused_lmhead_logprobs", "leap_selftest_bounded_wait",
 )
 LEAP_NOALLOC_MAX_ROWS = 65536
 
@@ -70,7 +71,9 @@ class RankStats(ctypes.Structure):
                 ("nonzero_adv_rollouts", ctypes.c_int64), ("first_turn_passes", ctypes.c_int64),
                 ("later_passes", ctypes.c_int64), ("groups_with_recovery", ctypes.c_int64),
                 ("failed_first_turn_in_gated", ctypes.c_int64), ("total_turns", ctypes.c_int64),
-                ("passes_by_turn", ctypes.c_int64 * 8)]
+                ("passes_by_turn", ctypes.c_int64 * 8),
+                ("composition", ctypes.c_int64 * (LEAP_PASS_BUCKETS * 3 * 2)),
+                ("groups_by_bucket", ctypes.c_int64 * LEAP_PASS_BUCKETS)]
 
 
 class LossParams(ctypes.Structure):
@@ -130,6 +133,8 @@ def lib() -> ctypes.CDLL:
     L.leap_fused_lmhead_logprobs.restype = S
     L.leap_fused_lmhead_logprobs.argtypes = [ctypes.POINTER(LossParams), _P, _P, _I64, _I32, _I32, _P, _P, _P, _P,
                                              _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]
+    L.leap_selftest_bounded_wait.restype = S
+    L.leap_selftest_bounded_wait.argtypes = [ctypes.c_uint64, _P, _P]
     L.leap_grpo_loss_bwd.restype = S
     L.leap_grpo_loss_bwd.argtypes = [ctypes.POINTER(LossParams), _P, _I64, _P, _P, _P, _P, _P, _I64, _I32,
                                      _P, _P]
@@ -433,7 +438,22 @@ def rank_stats_tensor(device):
 
 
 def read_rank_stats(t) -> dict:
+    """The counters as a dict; 'composition' is nested [bucket][type][sign]."""
     s = RankStats.from_buffer_copy(bytes(t.cpu().numpy().tobytes()))
-    d = {k: getattr(s, k) for k, _ in RankStats._fields_ if k != "passes_by_turn"}
+    arrays = ("passes_by_turn", "composition", "groups_by_bucket")
+    d = {k: getattr(s, k) for k, _ in RankStats._fields_ if k not in arrays}
     d["passes_by_turn"] = list(s.passes_by_turn)
+    flat = list(s.composition)
+    d["composition"] = [[flat[(b * 3 + k) * 2:(b * 3 + k) * 2 + 2] for k in range(3)]
+                        for b in range(LEAP_PASS_BUCKETS)]
+    d["groups_by_bucket"] = list(s.groups_by_bucket)
     return d
+
+
+def leap_selftest_bounded_wait(limit_ns, waited=None, stream=None):
+    """Runs the bounded-wait self-test kernel (a wait that can never complete,
+    given up after limit_ns); `waited` (uint64 device tensor of one element,
+    optional) receives the nanoseconds the wait took."""
+    st = lib().leap_selftest_bounded_wait(int(limit_ns), _ptr(waited), _stream(stream))
+    _check(st, "leap_selftest_bounded_wait")
+    return waited

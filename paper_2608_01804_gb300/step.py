@@ -8,7 +8,8 @@ stream:
   4. leap_scatter_turn_advantages  per-token advantage and aggregation weight
   5. leap_grpo_loss_fwd            clipped surrogate + fused dlogits (Eq. 3)
 Only step 3 leaves libleap, and only when a process group with more than one
-rank is passed in.  capture() records steps 1-5 as one CUDA graph for
+rank is passed in.  run() takes resident logits, run_chunked() a stream that
+exists chunk by chunk, run_streamed() logits in pinned host memory.  capture() records steps 1-5 as one CUDA graph for
 batches small enough that launching six kernels one by one costs more than
 running them.
 """
@@ -64,7 +65,12 @@ class GrpoStep:
         L.leap_rollout_token_counts(b.N, self.seg_offsets, self.seg_rollout, self.seg_turn,
                                     self.rank_out["T_eff"], M=b.M, L=self.L, totals=self.totals)
         if pg is not None and torch.distributed.get_world_size(pg) > 1:
-            torch.distributed.all_reduce(self.totals, group=pg)
+            if torch.distributed.get_backend(pg) == "nccl":
+                torch.distributed.all_reduce(self.totals, group=pg)
+            else:   # a host backend (gloo): the two counters travel through host memory
+                host = self.totals.cpu()
+                torch.distributed.all_reduce(host, group=pg)
+                self.totals.copy_(host)
         L.leap_scatter_turn_advantages(b.N, self.seg_offsets, self.seg_rollout, self.seg_turn,
                                        self.rank_out["turn_adv"], self.rank_out["T_eff"], self.L, self.totals,
                                        M=b.M, agg=self.agg, adv=self.adv, w=self.w)
@@ -80,6 +86,21 @@ class GrpoStep:
         """The whole pass for a batch whose logits are all resident."""
         self.advantages(pg)
         self.loss_pass(logits, ids, old_logp, dlogits)
+        return self.loss
+
+    def run_chunked(self, chunks, ids, old_logp, pg=None):
+        """The whole pass for a packed stream whose logits exist one chunk at a
+        time (a stream longer than HBM holds, e.g. the forward pass producing
+        the logits chunk by chunk).  `chunks` yields (row0, logits, dlogits):
+        consecutive row ranges [row0, row0 + logits.shape[0]) that cover the
+        stream in order; ids and old_logp are device tensors of all rows.  The
+        advantages and weights are computed once for the whole stream, then
+        the fused loss runs chunk by chunk, accumulating the loss."""
+        self.advantages(pg)
+        for c, (row0, z, dl) in enumerate(chunks):
+            n = z.shape[0]
+            self._ensure_workspace(n)
+            self.loss_pass(z, ids[row0:row0 + n], old_logp[row0:row0 + n], dl, row0=row0, accumulate=c > 0)
         return self.loss
 
     def capture(self, logits, ids, old_logp, dlogits, warmup=2):
@@ -118,6 +139,7 @@ class GrpoStep:
         if not host_logits.is_pinned():
             raise ValueError("host_logits must be in pinned host memory")
         N, ld = host_logits.shape
+        self._ensure_workspace(min(N, chunk_rows))
         comp = torch.cuda.current_stream(self.dev)
         cs = self._copy_stream()
         staging = self._staging(chunk_rows, ld, host_logits.dtype)
@@ -141,6 +163,12 @@ class GrpoStep:
             done.record(comp)
             free[c % 2] = done
         return self.loss
+
+    def _ensure_workspace(self, rows):
+        """Grows the loss workspace to cover `rows` rows per loss call."""
+        need = L.leap_grpo_loss_workspace_size(rows, self.V)
+        if self.workspace.numel() < need:
+            self.workspace = L.loss_workspace(rows, self.V, self.dev)
 
     def _copy_stream(self):
         if getattr(self, "_cs", None) is None:

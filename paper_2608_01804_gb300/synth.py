@@ -108,15 +108,18 @@ def single_turn_batch(seed=1, num_prompts=16):
 
 
 def multiturn_dcp_batch(seed=2, num_prompts=32, G=16, M=3, len_lo=256, len_hi=2048, frac_expanded=0.4,
-                        tau=(8, 15), later_pass_prob=0.35):
+                        tau=(8, 15), later_pass_prob=0.35, prompt_lo=256, prompt_hi=1024):
     """Packed ragged multi-turn batch (the DCP workload).
 
     A fraction `frac_expanded` of prompts is drawn as multi-turn: their
     first-turn failure count is uniform in [tau[0], tau[1]]; the others draw it
     outside that zone.  In expanded groups each first-turn failure receives an
     environment-feedback segment and another turn, up to M, passing each later
-    turn with probability `later_pass_prob`.  Generated turns and feedback
-    segments are U{len_lo..len_hi} tokens, packed back to back.
+    turn with probability `later_pass_prob`.  Each rollout's packed sequence
+    starts with its prompt (U{prompt_lo..prompt_hi} tokens, one length per
+    prompt, shared by its G rollouts; prompt_hi = 0 leaves prompts out), then
+    its turns; generated turns and feedback segments are U{len_lo..len_hi}
+    tokens.  Prompt and feedback tokens are masked segments (turn -1).
     """
     rng = np.random.default_rng(seed)
     n = num_prompts * G
@@ -147,12 +150,18 @@ def multiturn_dcp_batch(seed=2, num_prompts=32, G=16, M=3, len_lo=256, len_hi=20
                         break
                     t += 1
     speed = rng.lognormal(0.0, 0.5, size=n).astype(np.float32)
+    prompt_len = (rng.integers(prompt_lo, prompt_hi + 1, size=num_prompts) if prompt_hi > 0
+                  else np.zeros(num_prompts, dtype=np.int64))
     segs = []
     ntok = np.zeros(n, dtype=np.int32)
     starts = np.zeros(n + 1, dtype=np.int64)
     cur = 0
     for i in range(n):
         starts[i] = cur
+        pl = int(prompt_len[i // G])
+        if pl > 0:
+            segs.append((pl, -1, -1))
+            cur += pl
         for t in range(int(num_turns[i])):
             if t > 0:
                 fb = int(rng.integers(len_lo, len_hi + 1))

@@ -73,3 +73,4 @@ def test_host_argument_checks_need_no_gpu():
                                   ctypes.c_void_p(256), None, None, None, None, ctypes.c_void_p(256), 16,
                                   None, None) == L.LEAP_ERR_INVALID_ARG
     assert lib.leap_grpo_loss_workspace_size(4096, 151936) >= 4096 * 13
+    assert lib.leap_selftest_bounded_wait(10, None, None) == L.LEAP_ERR_INVALID_ARG   # limit below 1 us

@@ -86,6 +86,33 @@ def test_single_turn_workload_full_size_sampled():
     assert torch.all(out["dlogits"][masked] == 0)
 
 
+def test_single_turn_whole_batch_loss_against_oracle():
+    """The benchmark's whole-batch loss (32,768 rows at V = 151,936, 21,662 of
+    them valid) against the oracle's fp64 loss over every valid row, computed
+    on the host 512 rows at a time (3.3 G fp64 log-softmax terms)."""
+    L = leap()
+    b = synth.single_turn_batch()
+    V = 151936
+    z = synth.logits(b.N, V, 3.0, 200, "cuda", spike_frac=0.01)
+    ids = synth.token_ids(b.N, V, 201, "cuda")
+    old = torch_logp(z, ids, V) + synth.normal(b.N, 0.05, 202, "cuda")
+    _, _, _, out = _gpu_pipeline(L, b, z, ids, old, V, 1.0, (0, b.G), False)
+    loss = out["loss"].item()
+    del out
+    _, adv_o, w_o = _oracle_pipeline(b, 1.0, (0, b.G), False)
+    live = np.nonzero(w_o)[0]
+    assert len(live) == 21662
+    ids_h = ids.cpu().numpy().astype(np.int64)
+    old_h = old.cpu().numpy().astype(np.float64)
+    total = 0.0
+    for a in range(0, len(live), 512):
+        rows = live[a:a + 512]
+        res = O.grpo_loss_rows(rows_f64(z, rows, V), ids_h[rows], old_h[rows], adv_o[rows], w_o[rows],
+                               want_dlogits=False)
+        total += res["loss"]
+    assert abs(loss - total) <= TOL_LOSS_REL * abs(total), (loss, total)
+
+
 def test_multiturn_dcp_workload_chunked():
     """The packed multi-turn batch (~1M tokens) streamed through one 65,536-row
     logits chunk buffer with loss accumulation; three chunks are checked against
@@ -160,6 +187,13 @@ def test_streamed_step_equals_resident_step():
     assert loss_str.item() == expect.item()
     # The whole-batch loss differs from the chunked one only by the fp32 sum over chunks.
     assert abs(loss_str.item() - loss_res.item()) <= 4 * 2.0 ** -24 * float(step.w.abs().sum().item()) * 2.0
+    # A step built for smaller chunks grows its workspace for the streamed chunk size.
+    small = GrpoStep(b, V, "cuda", gamma=1.0, tau=(0, b.G), use_gate_in=False, chunk_rows=256)
+    dl_small = torch.full_like(z, 7)
+    loss_small = small.run_streamed(host, ids, old, dl_small, chunk_rows=1500).clone()
+    torch.cuda.synchronize()
+    assert loss_small.item() == loss_str.item()
+    assert torch.equal(dl_small, dl_res)
 
 
 def test_graph_replay_equals_eager_step():

@@ -197,6 +197,29 @@ def test_rank_stats_full_size_tournament():
     assert L.read_rank_stats(st) == O.rank_stats(orc, pt.reshape(-1, G), M)
 
 
+@pytest.mark.parametrize("G,M,groups,reward,tau", [(64, 3, 65536, 0, (20, 44)), (64, 3, 65536, 1, (20, 44)),
+                                                    (33, 2, 4000, 0, (10, 25)), (100, 3, 2000, 1, (30, 80)),
+                                                    (8, 1, 8000, 0, (0, 8))])
+def test_rank_composition_matches_oracle(G, M, groups, reward, tau):
+    """Fig. 4 counters (pass-rate bucket x outcome type x sign of A) and the
+    other training counters, pair kernel and generic kernel, tournament and
+    static-scalar rewards (the two reward definitions the figure compares),
+    equal to the oracle."""
+    pt, nt, _, _ = synth.tournament_outcomes(seed=G + M, num_groups=groups, G=G, M=M)
+    L = leap()
+    st = L.rank_stats_tensor("cuda")
+    L.leap_group_rank_advantages(to_dev(pt, torch.int8), to_dev(nt, torch.int8), G=G, M=M, tau_min=tau[0],
+                                 tau_max=tau[1], gamma=0.9, stats=st, reward=reward, static_c=0.5)
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, tau[0], tau[1], 0.9, reward=reward,
+                            static_c=0.5)
+    exp = O.rank_stats(orc, pt.reshape(-1, G), M)
+    got = L.read_rank_stats(st)
+    assert got["composition"] == exp["composition"]
+    assert got["groups_by_bucket"] == exp["groups_by_bucket"]
+    assert got == exp
+    assert sum(sum(sum(x) for x in b) for b in got["composition"]) == got["nonzero_adv_rollouts"]
+
+
 @pytest.mark.parametrize("G,M", [(64, 3), (16, 2), (2, 8)])
 def test_pair_and_generic_kernels_agree(G, M):
     """Even G <= 64 with the paper's comparator runs the pair kernel (vector
