@@ -397,6 +397,7 @@ def multiturn_step(device, peak, steps=3, warmup=1):
         step.run_chunked(chunks, ids, old)
     torch.cuda.synchronize()
     live = int((step.w != 0).sum().item())
+    tok_launches = step.token_launches()
     stream = torch.cuda.current_stream()
     a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     a_ev.record(stream)
@@ -409,7 +410,7 @@ def multiturn_step(device, peak, steps=3, warmup=1):
     gbs = alg / (ms / 1e3) / 1e9
     out = {"ms_per_step": ms, "rows": N, "valid_tokens": live, "chunks": len(chunks), "algorithmic_bytes": alg,
            "achieved_gbs": gbs, "frac": gbs / peak, "throughput": live / (ms / 1e3), "unit": "valid tokens/s",
-           "launches_per_step": 1 + (1 if b.n <= GrpoStep.ONE_BLOCK_COUNT_ROLLOUTS else 3) + 1 + 3 * len(chunks),
+           "launches_per_step": 1 + tok_launches + 3 * len(chunks),
            "note": "whole step (rank, counts, scatter, fused loss + reductions per chunk); one 65,536-row "
                    "logits chunk reused for every chunk"}
     del zbuf, dlbuf, step
@@ -481,6 +482,27 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
         L.leap_scatter_turn_advantages(b.N, so, sr, st_, rk["turn_adv"], rk["T_eff"], Lc, tot, M=b.M, adv=adv, w=w)
     ms = _timed_launches(tok, reps * 4, stream, flush, lead_cycles=LEAD_CYCLES)
     rows["token_counts_scatter_multiturn_%d_tokens" % b.N] = entry(8 * b.N, ms, b.N, "tokens/s")
+    fused = lambda: L.leap_token_advantages(b.N, so, sr, st_, rk["turn_adv"], rk["T_eff"], M=b.M, L=Lc, totals=tot,
+                                            adv=adv, w=w)
+    ms = _timed_launches(fused, reps * 4, stream, flush, lead_cycles=LEAD_CYCLES)
+    rows["token_advantages_one_launch_multiturn_%d_tokens" % b.N] = entry(8 * b.N, ms, b.N, "tokens/s")
+    # The same two ways on the small workload's padded layout (16,384 tokens).
+    tbk = synth.tiny_batch()
+    t_so, t_sr, t_st = (torch.as_tensor(x).to(device) for x in (tbk.seg_offsets, tbk.seg_rollout, tbk.seg_turn))
+    t_rk = L.leap_group_rank_advantages(torch.as_tensor(tbk.pass_turn).to(device),
+                                        torch.as_tensor(tbk.num_turns).to(device), G=tbk.G, M=tbk.M, gamma=0.9)
+    t_L, t_tot, t_adv, t_w = L.leap_token_advantages(tbk.N, t_so, t_sr, t_st, t_rk["turn_adv"], t_rk["T_eff"], M=tbk.M)
+
+    def t_two():
+        L.leap_rollout_token_counts(tbk.N, t_so, t_sr, t_st, t_rk["T_eff"], M=tbk.M, L=t_L, totals=t_tot)
+        L.leap_scatter_turn_advantages(tbk.N, t_so, t_sr, t_st, t_rk["turn_adv"], t_rk["T_eff"], t_L, t_tot,
+                                       M=tbk.M, adv=t_adv, w=t_w)
+    t_one = lambda: L.leap_token_advantages(tbk.N, t_so, t_sr, t_st, t_rk["turn_adv"], t_rk["T_eff"], M=tbk.M,
+                                            L=t_L, totals=t_tot, adv=t_adv, w=t_w)
+    ms = _timed_launches(t_two, reps * 4, stream, flush, lead_cycles=LEAD_CYCLES)
+    rows["token_counts_scatter_tiny_%d_tokens" % tbk.N] = entry(8 * tbk.N, ms, tbk.N, "tokens/s")
+    ms = _timed_launches(t_one, reps * 4, stream, flush, lead_cycles=LEAD_CYCLES)
+    rows["token_advantages_one_launch_tiny_%d_tokens" % tbk.N] = entry(8 * tbk.N, ms, tbk.N, "tokens/s")
     del adv, w
 
     # The whole pass on the multi-turn DCP workload (a1-a7 over the chunked stream).
@@ -686,9 +708,16 @@ def tokens_only(args):
         tok()
     ms = _timed_launches(tok, args.steps, torch.cuda.current_stream(), lambda: flush_buf.fill_(1),
                          lead_cycles=LEAD_CYCLES)
+    one = lambda: L.leap_token_advantages(b.N, so, sr, st_, rk["turn_adv"], rk["T_eff"], M=b.M, L=Lc, totals=tot,
+                                          adv=adv, w=w)
+    for _ in range(args.warmup):
+        one()
+    ms1 = _timed_launches(one, args.steps, torch.cuda.current_stream(), lambda: flush_buf.fill_(1),
+                          lead_cycles=LEAD_CYCLES)
     peak, _ = measured_peaks()
     print(json.dumps({"tokens": b.N, "segments": int(b.seg_rollout.size), "ms": ms, "gbs": 8 * b.N / ms / 1e6,
-                      "frac": 8 * b.N / ms / 1e6 / peak}), flush=True)
+                      "frac": 8 * b.N / ms / 1e6 / peak, "one_launch_ms": ms1,
+                      "one_launch_frac": 8 * b.N / ms1 / 1e6 / peak}), flush=True)
 
 
 def short_rows(args):
@@ -930,7 +959,7 @@ def main():
                            "vocab": V, "logits_dtype": "bf16", "l2": "inputs larger than L2 (9.96 GB of logits "
                            "read and 9.96 GB of dlogits written per step)", "parallelism": "dp%d" % world},
                 "roofline": roofline, "rows": rows, "cpu_baseline": cpu, "e2e": e2e,
-                "gpu_launches": K * step.launches_per_run(), "clocks": clk}
+                "gpu_launches": K * step.launches_per_run(pg), "clocks": clk}
         print(json.dumps(line), flush=True)
     if pg is not None:
         torch.distributed.destroy_process_group()

@@ -225,6 +225,26 @@ leap_status_t leap_scatter_turn_advantages(
     float* adv_out, float* w_out,
     void* stream);
 
+/*
+ * leap_rollout_token_counts followed by leap_scatter_turn_advantages with
+ * this call's own totals (no exchange in between), in one launch: every block
+ * builds the counts and each segment's advantage and weight in shared memory,
+ * then scatters its share of the tokens.  Same arguments and results as the
+ * two calls (L, totals, adv_out, w_out written; malformed segments flagged
+ * and skipped alike).  For one process (or one rank holding the whole batch).
+ * When the batch is split over data-parallel ranks the totals must be
+ * all-reduced between counting and scattering: use the two calls.  The one
+ * launch serves tables of up to 768 segments (every block rebuilds the table,
+ * which pays off on small batches only); larger ones take the two calls'
+ * kernels.
+ */
+leap_status_t leap_token_advantages(
+    int64_t N, int32_t n_rollouts, int32_t M,
+    const int32_t* seg_offsets, const int32_t* seg_rollout, const int8_t* seg_turn,
+    int32_t num_segs, const float* turn_adv, const uint8_t* T_eff, int32_t agg,
+    int32_t* L, int64_t* totals, float* adv_out, float* w_out,
+    void* stream);
+
 /* ------------------------------------------------------------------------
  * 3. Token log-probabilities under pi_theta (the log pi terms of Eq. 3's
  *    surrogate): lse_k = log sum_v exp(inv_temp * z_kv),

@@ -219,6 +219,34 @@ leap_status_t leap_scatter_turn_advantages(int64_t N, int32_t n_rollouts, int32_
     return from_cuda(launch_scatter(a, static_cast<cudaStream_t>(stream)));
 }
 
+leap_status_t leap_token_advantages(int64_t N, int32_t n_rollouts, int32_t M, const int32_t* seg_offsets,
+                                    const int32_t* seg_rollout, const int8_t* seg_turn, int32_t num_segs,
+                                    const float* turn_adv, const uint8_t* T_eff, int32_t agg, int32_t* L,
+                                    int64_t* totals, float* adv_out, float* w_out, void* stream) {
+    if (!seg_args_ok(N, n_rollouts, M, seg_offsets, seg_rollout, seg_turn, num_segs, T_eff)) return LEAP_ERR_INVALID_ARG;
+    if (agg != LEAP_AGG_SEQ_MEAN_TOKEN_MEAN && agg != LEAP_AGG_TOKEN_MEAN) return LEAP_ERR_INVALID_ARG;
+    if (!totals || (n_rollouts > 0 && (!L || !turn_adv)) || (N > 0 && (!adv_out || !w_out)))
+        return LEAP_ERR_INVALID_ARG;
+    SegArgs a = {};
+    a.N = N;
+    a.n_rollouts = n_rollouts;
+    a.M = M;
+    a.num_segs = num_segs;
+    a.seg_offsets = seg_offsets;
+    a.seg_rollout = seg_rollout;
+    a.seg_turn = seg_turn;
+    a.T_eff = T_eff;
+    a.turn_adv = turn_adv;
+    a.L_out = L;
+    a.totals_out = totals;
+    a.agg = agg;
+    a.adv_out = adv_out;
+    a.w_out = w_out;
+    a.status = status_ptr();
+    if (!a.status) return LEAP_ERR_CUDA;
+    return from_cuda(launch_token_advantages(a, static_cast<cudaStream_t>(stream)));
+}
+
 leap_status_t leap_token_logprobs(const uint16_t* logits, int64_t ld, const int32_t* ids, int64_t N, int32_t V,
                                   float inv_temp, float* logp, float* lse, void* stream) {
     if (!rows_ok(logits, ld, ids, N, V)) return LEAP_ERR_INVALID_ARG;

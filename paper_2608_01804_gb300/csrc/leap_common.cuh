@@ -209,6 +209,12 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity
     return mbar_wait_bounded<true>(bar, parity, status, abort_flag);
 }
 
+// Orders this thread's earlier generic-proxy accesses of shared memory before
+// later async-proxy ones (a bulk copy into a buffer it has just read).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // 1-D bulk copy global -> own shared memory, completing on `bar` (bytes and
 // both addresses multiples of 16).
 __device__ __forceinline__ void bulk_g2s(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_t* bar) {

@@ -89,6 +89,9 @@ LossWorkspace carve_loss_workspace(void* base, int64_t N);
 cudaError_t launch_rank_advantages(const RankArgs& a, cudaStream_t s);
 cudaError_t launch_token_counts(const SegArgs& a, cudaStream_t s);
 cudaError_t launch_scatter(const SegArgs& a, cudaStream_t s);
+// Counts (to L_out, totals_out) and scatter with those local totals, in one
+// launch when the segment table fits on chip.
+cudaError_t launch_token_advantages(const SegArgs& a, cudaStream_t s);
 
 // mode: 0 = log-probs only, 1 = loss forward (no dlogits).
 cudaError_t launch_row_stream(const RowArgs& a, int mode, cudaStream_t s);

@@ -521,6 +521,146 @@ __global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs
     if (a.stats) flush_stats(a, sst);
 }
 
+// G = 64 with the paper's comparator and the tournament reward, without
+// counters: a warp takes two groups per iteration (128 consecutive rollouts),
+// lane l holding rollouts 4l .. 4l + 3 (lanes 0-15 the first group, 16-31 the
+// second).  Each outcome array is one 4-byte load and each output array one
+// 16-byte store per lane (the turn advantages as M float4), and the two
+// groups' sums share warp reductions (the failure counts packed in 16-bit
+// halves, the tier histograms and squared net scores one reduction per group):
+// half the memory instructions and loop overhead of the pair kernel per
+// rollout.
+constexpr int kQuadMinBlocks = 4;
+template <int MC>
+__global__ void __launch_bounds__(256, kQuadMinBlocks) rank_quad_kernel(RankArgs a) {
+    constexpr int J = 4, M = MC, G = 64;
+    const int lane = threadIdx.x & 31;
+    const int half = lane >> 4;
+    const int64_t npairs = ((int64_t)a.num_groups + 1) / 2;
+    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    for (int64_t pr = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); pr < npairs; pr += warps) {
+        const int64_t group = 2 * pr + half;
+        const bool own = group < a.num_groups;   // the last pair may hold one group
+        const int64_t i0 = group * G + 4 * (lane & 15);
+        int pt[J], T[J];
+        {
+            unsigned p4 = 0u, n4 = 0x01010101u;
+            if (own) {
+                p4 = *reinterpret_cast<const uint32_t*>(a.pass_turn + i0);
+                n4 = *reinterpret_cast<const uint32_t*>(a.num_turns + i0);
+            }
+#pragma unroll
+            for (int j = 0; j < J; ++j) {
+                pt[j] = (int8_t)((p4 >> (8 * j)) & 0xffu);
+                T[j] = (int8_t)((n4 >> (8 * j)) & 0xffu);
+            }
+        }
+        bool valid[J], bad[J];
+        int pt0[J], r[J];
+        int fails = 0;
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            valid[j] = own;
+            bool fail1;
+            decode_outcome(pt[j], T[j], M, valid[j], bad[j], fail1, pt0[j]);
+            fails += fail1;
+        }
+        const unsigned both = __reduce_add_sync(0xffffffffu, (unsigned)fails << (16 * half));
+        const int n_fail = (int)(half ? (both >> 16) : (both & 0xffffu));
+        const bool gate = a.gate_in ? (own && a.gate_in[group] != 0) : (a.tau_min <= n_fail && n_fail <= a.tau_max);
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            tier_rule(pt0[j], T[j], valid[j], bad[j], gate, M, r[j], T[j]);
+            if (bad[j]) flag_status(a.status, 2u);
+        }
+
+        // Eq. 5: the tier histogram of each group (8-bit counters, four tiers
+        // to a word), then the byte-wise prefix as in the pair kernel.
+        constexpr int W = (M + 4) / 4;
+        unsigned hist[W], pre[W];
+#pragma unroll
+        for (int w = 0; w < W; ++w) {
+            unsigned mine = 0;
+#pragma unroll
+            for (int j = 0; j < J; ++j)
+                if (own && (r[j] >> 2) == w) mine += 1u << (8 * (r[j] & 3));
+            const unsigned h0 = __reduce_add_sync(0xffffffffu, half ? 0u : mine);
+            const unsigned h1 = __reduce_add_sync(0xffffffffu, half ? mine : 0u);
+            hist[w] = half ? h1 : h0;
+        }
+        unsigned carry = 0;
+#pragma unroll
+        for (int w = 0; w < W; ++w) {
+            pre[w] = hist[w] * 0x01010101u + carry * 0x01010101u;
+            carry = pre[w] >> 24;
+        }
+        const int below = (int)carry;   // == G
+        int nw[J], nb[J], d[J];
+        int dsq = 0;
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            const int w = r[j] >> 2, k = r[j] & 3;
+            unsigned hw = hist[0], pw = pre[0];
+#pragma unroll
+            for (int q = 1; q < W; ++q)
+                if (w == q) {
+                    hw = hist[q];
+                    pw = pre[q];
+                }
+            const int eq = (int)((hw >> (8 * k)) & 0xffu);
+            const int incl = (int)((pw >> (8 * k)) & 0xffu);
+            nw[j] = incl - eq;
+            nb[j] = below - incl;
+            d[j] = nw[j] - nb[j];
+            dsq += d[j] * d[j];
+        }
+        if (!own) dsq = 0;
+        const int dd0 = __reduce_add_sync(0xffffffffu, half ? 0 : dsq);
+        const int dd1 = __reduce_add_sync(0xffffffffu, half ? dsq : 0);
+        const int dd = half ? dd1 : dd0;
+
+        float Rv[J], Av[J];
+        group_reward<J>(a, G, M, d, r, valid, dd, Rv, Av);
+
+        if (own) {
+            if (a.n_worse) *reinterpret_cast<int4*>(a.n_worse + i0) = make_int4(nw[0], nw[1], nw[2], nw[3]);
+            if (a.n_better) *reinterpret_cast<int4*>(a.n_better + i0) = make_int4(nb[0], nb[1], nb[2], nb[3]);
+            if (a.r_out)
+                *reinterpret_cast<uint32_t*>(a.r_out + i0) =
+                    (uint32_t)r[0] | ((uint32_t)r[1] << 8) | ((uint32_t)r[2] << 16) | ((uint32_t)r[3] << 24);
+            *reinterpret_cast<uint32_t*>(a.T_eff + i0) =
+                (uint32_t)T[0] | ((uint32_t)T[1] << 8) | ((uint32_t)T[2] << 16) | ((uint32_t)T[3] << 24);
+            if (a.R) *reinterpret_cast<float4*>(a.R + i0) = make_float4(Rv[0], Rv[1], Rv[2], Rv[3]);
+            if (a.A) *reinterpret_cast<float4*>(a.A + i0) = make_float4(Av[0], Av[1], Av[2], Av[3]);
+            // Sec. 3.3: beta = gamma for A >= 0, else 1; the last counted turn keeps A.
+            float tv[J * M];
+#pragma unroll
+            for (int j = 0; j < J; ++j) {
+                const float beta = (Av[j] >= 0.f) ? a.gamma : 1.f;
+                float p = Av[j];
+#pragma unroll
+                for (int t = M - 1; t >= 0; --t) {
+                    tv[j * M + t] = (t < T[j]) ? p : 0.f;
+                    if (t < T[j]) p *= beta;
+                }
+            }
+            float4* ta = reinterpret_cast<float4*>(a.turn_adv + i0 * M);
+#pragma unroll
+            for (int q = 0; q < M; ++q) ta[q] = make_float4(tv[4 * q], tv[4 * q + 1], tv[4 * q + 2], tv[4 * q + 3]);
+            if ((lane & 15) == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
+        }
+    }
+}
+
+template <int MC>
+cudaError_t launch_quad(const RankArgs& a, cudaStream_t s) {
+    const int warps = 8;
+    const int64_t pairs = ((int64_t)a.num_groups + 1) / 2;
+    const int64_t blocks = std::min<int64_t>((pairs + warps - 1) / warps, (int64_t)device_sm_count() * kQuadMinBlocks);
+    rank_quad_kernel<MC><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
 template <int J>
 cudaError_t launch_rank_j(const RankArgs& a, cudaStream_t s) {
     const int warps = 8;
@@ -718,6 +858,150 @@ __global__ void __launch_bounds__(256) scatter_kernel(SegArgs a) {
     }
 }
 
+// ---- counts + scatter in one launch (single rank) ---------------------------
+// Every block builds in shared memory what the scatter needs from the whole
+// batch: the per-rollout counts L (hence the two totals), then for every
+// segment its advantage, weight and the end of its weighted tokens; then its
+// warps scatter their 256-token chunks with the same 32-ary search and walk
+// as scatter_kernel, reading the segment table from shared memory instead of
+// chasing dependent global loads.  Block 0 also writes L and the totals.  The
+// counting is repeated by every block (a few KB of the segment table read from
+// L2 per block) in exchange for one launch instead of two.
+constexpr int kTokThreads = 256;
+// Every block repeats the table work, so the one launch pays off on small
+// tables only (measured: 117 / 255 segments 0.75 / 0.71 of the two launches'
+// time; 1,514 segments 1.32 times it).
+constexpr int kTokMaxSegs = 768;
+constexpr size_t kTokSmemMax = 48 * 1024;
+
+size_t fused_tok_smem(int64_t n, int64_t S) { return 4 * (size_t)n + 4 * ((size_t)S + 1) + 12 * (size_t)S; }
+
+__global__ void __launch_bounds__(kTokThreads) token_adv_fused_kernel(SegArgs a) {
+    extern __shared__ __align__(16) int32_t tsm[];
+    const int n = a.n_rollouts, S = a.num_segs;
+    int32_t* sL = tsm;                                    // [n] per-rollout counts
+    int32_t* soff = sL + n;                               // [S + 1] segment offsets
+    int32_t* send = soff + S + 1;                         // [S] end of the weighted tokens (= start if none)
+    float* sadv = reinterpret_cast<float*>(send + S);     // [S]
+    float* sw = sadv + S;                                 // [S]
+    __shared__ long long red[2][kTokThreads / 32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+
+    for (int i = tid; i < n; i += kTokThreads) sL[i] = 0;
+    if (S > 0)
+        for (int q = tid; q <= S; q += kTokThreads) soff[q] = a.seg_offsets[q];
+    __syncthreads();
+    auto seg_fields = [&](int q, int& lo, int& hi, int& i, int& t) {
+        lo = soff[q];
+        hi = soff[q + 1];
+        t = a.seg_turn[q];
+        i = a.seg_rollout[q];
+        return lo >= 0 && hi >= lo && (int64_t)hi <= a.N && t < a.M && (t < 0 || (i >= 0 && i < n));
+    };
+    for (int q = tid; q < S; q += kTokThreads) {   // L_i (Sec. 3.3 token sets)
+        int lo, hi, i, t;
+        if (!seg_fields(q, lo, hi, i, t)) {
+            if (blockIdx.x == 0) flag_status(a.status, 4u);
+            continue;
+        }
+        if (t >= 0 && hi > lo && t < (int)a.T_eff[i]) atomicAdd(&sL[i], hi - lo);
+    }
+    __syncthreads();
+    long long tok = 0, roll = 0;
+    for (int i = tid; i < n; i += kTokThreads) {
+        const int32_t l = sL[i];
+        tok += l;
+        roll += (l > 0);
+        if (blockIdx.x == 0) a.L_out[i] = l;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        tok += __shfl_xor_sync(0xffffffffu, tok, o);
+        roll += __shfl_xor_sync(0xffffffffu, roll, o);
+    }
+    if (lane == 0) {
+        red[0][warp] = tok;
+        red[1][warp] = roll;
+    }
+    __syncthreads();
+    long long nv = 0, rv = 0;
+#pragma unroll
+    for (int k = 0; k < kTokThreads / 32; ++k) {
+        nv += red[0][k];
+        rv += red[1][k];
+    }
+    if (blockIdx.x == 0 && tid == 0) {
+        a.totals_out[0] = nv;
+        a.totals_out[1] = rv;
+    }
+    for (int q = tid; q < S; q += kTokThreads) {   // per-segment advantage and weight
+        int lo, hi, i, t;
+        const bool ok = seg_fields(q, lo, hi, i, t);
+        float av = 0.f, wv = 0.f;
+        int end = lo;
+        if (ok && t >= 0 && t < (int)a.T_eff[i]) {
+            av = a.turn_adv[(int64_t)i * a.M + t];
+            if (a.agg == 1) {
+                wv = nv > 0 ? recip_count((double)nv) : 0.f;
+            } else {
+                const int32_t Li = sL[i];
+                wv = (rv > 0 && Li > 0) ? recip_count((double)rv * (double)Li) : 0.f;
+            }
+            end = hi;
+        }
+        send[q] = end;
+        sadv[q] = av;
+        sw[q] = wv;
+    }
+    __syncthreads();
+
+    const int64_t chunk = (int64_t)32 * kScatterIters;
+    const int64_t nchunks = (a.N + chunk - 1) / chunk;
+    const int64_t warps = (int64_t)gridDim.x * (kTokThreads / 32);
+    for (int64_t c = (int64_t)blockIdx.x * (kTokThreads / 32) + warp; c < nchunks; c += warps) {
+        const int64_t k0 = c * chunk;
+        int32_t seg = 0;   // last s with soff[s] <= k0 (0 if none), 32-ary search
+        if (S > 0) {
+            int32_t lo = 0, cnt = S;
+            while (cnt > 1) {
+                const int32_t step = (cnt + 31) / 32;
+                const bool in = lane * step < cnt;
+                const bool le = in && soff[lo + lane * step] <= k0;
+                const unsigned m = __ballot_sync(0xffffffffu, le);
+                if (m == 0) break;
+                const int32_t hl = 31 - __clz(m);
+                lo += hl * step;
+                cnt = min(step, cnt - hl * step);
+            }
+            seg = lo;
+        }
+        int32_t cur = -1, clo = 0, chi = 0;
+        float cadv = 0.f, cw = 0.f;
+#pragma unroll 1
+        for (int it = 0; it < kScatterIters; ++it) {
+            const int64_t k = k0 + it * 32 + lane;
+            if (k >= a.N) break;
+            float adv = 0.f, w = 0.f;
+            if (S > 0) {
+                while (seg + 1 < S && soff[seg + 1] <= k) ++seg;
+                if (seg != cur) {
+                    cur = seg;
+                    clo = soff[seg];
+                    chi = send[seg];
+                    cadv = sadv[seg];
+                    cw = sw[seg];
+                }
+                if (k >= clo && k < chi) {
+                    adv = cadv;
+                    w = cw;
+                }
+            }
+            a.adv_out[k] = adv;
+            a.w_out[k] = w;
+        }
+    }
+}
+
 bool aligned_to(const void* p, uintptr_t n) { return (reinterpret_cast<uintptr_t>(p) & (n - 1)) == 0; }
 
 template <int MC>
@@ -735,6 +1019,25 @@ cudaError_t launch_pair(const RankArgs& a, cudaStream_t s) {
 
 cudaError_t launch_rank_advantages(const RankArgs& a, cudaStream_t s) {
     if (a.num_groups == 0) return cudaSuccess;
+    // Groups of 64 (the quad kernel): 4-byte aligned byte arrays and 16-byte
+    // aligned 4-byte arrays (every lane's four rollouts start at a multiple of 4).
+    const bool quad = a.cmp == 0 && a.reward == 0 && !a.stats && a.G == 64 && aligned_to(a.pass_turn, 4) &&
+                      aligned_to(a.num_turns, 4) && aligned_to(a.T_eff, 4) && aligned_to(a.r_out, 4) &&
+                      aligned_to(a.n_worse, 16) && aligned_to(a.n_better, 16) && aligned_to(a.R, 16) &&
+                      aligned_to(a.A, 16) && aligned_to(a.turn_adv, 16);
+    if (quad) {
+        switch (a.M) {
+            case 1: return launch_quad<1>(a, s);
+            case 2: return launch_quad<2>(a, s);
+            case 3: return launch_quad<3>(a, s);
+            case 4: return launch_quad<4>(a, s);
+            case 5: return launch_quad<5>(a, s);
+            case 6: return launch_quad<6>(a, s);
+            case 7: return launch_quad<7>(a, s);
+            case 8: return launch_quad<8>(a, s);
+            default: break;
+        }
+    }
     // The pair kernel's vector accesses need 2-byte aligned byte arrays and
     // 8-byte aligned 4-byte arrays (rollout pairs start at even indices).
     const bool pair = a.cmp == 0 && a.G % 2 == 0 && a.G <= 64 && aligned_to(a.pass_turn, 2) &&
@@ -777,6 +1080,24 @@ cudaError_t launch_token_counts(const SegArgs& a, cudaStream_t s) {
     if (a.n_rollouts > 0) {
         totals_kernel<<<(unsigned)std::max<int64_t>(zb, 1), 256, 0, s>>>(a.L_out, a.n_rollouts, a.totals_out);
     }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_token_advantages(const SegArgs& a, cudaStream_t s) {
+    const size_t smem = fused_tok_smem(a.n_rollouts, a.num_segs);
+    if (a.num_segs > kTokMaxSegs || smem > kTokSmemMax) {   // a large table: the two-kernel path
+        cudaError_t e = launch_token_counts(a, s);
+        if (e != cudaSuccess) return e;
+        SegArgs b = a;
+        b.L_in = a.L_out;
+        b.totals_in = a.totals_out;
+        return launch_scatter(b, s);
+    }
+    const int sms = device_sm_count();
+    const int64_t chunks = (a.N + 32 * kScatterIters - 1) / (32 * kScatterIters);
+    const int64_t wpb = kTokThreads / 32;
+    const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((chunks + wpb - 1) / wpb, (int64_t)sms * 2));
+    token_adv_fused_kernel<<<(unsigned)blocks, kTokThreads, smem, s>>>(a);
     return cudaGetLastError();
 }
 

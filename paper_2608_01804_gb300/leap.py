@@ -46,6 +46,7 @@ LEAP_PASS_BUCKETS = 10
 EXPORTS = (
     "leap_status_string", "leap_version", "leap_get_device_status",
     "leap_group_rank_advantages", "leap_rollout_token_counts", "leap_scatter_turn_advantages",
+    "leap_token_advantages",
     "leap_token_logprobs", "leap_grpo_loss_workspace_size", "leap_grpo_loss_fwd", "leap_grpo_loss_bwd",
     "leap_grpo_loss_fwd_noalloc", "leap_gemm_bf16_nt", "leap_gemm_bf16_tn_f32", "leap_fused_lmhead_workspace_size",
     "leap_fused_lmhead_logprobs", "leap_selftest_bounded_wait",
@@ -114,6 +115,8 @@ def lib() -> ctypes.CDLL:
     L.leap_scatter_turn_advantages.restype = S
     L.leap_scatter_turn_advantages.argtypes = [_I64, _I32, _I32, _P, _P, _P, _I32, _P, _P, _P, _P, _I32,
                                                _P, _P, _P]
+    L.leap_token_advantages.restype = S
+    L.leap_token_advantages.argtypes = [_I64, _I32, _I32, _P, _P, _P, _I32, _P, _P, _I32, _P, _P, _P, _P, _P]
     L.leap_token_logprobs.restype = S
     L.leap_token_logprobs.argtypes = [_P, _I64, _P, _I64, _I32, _F32, _P, _P, _P]
     L.leap_grpo_loss_workspace_size.restype = _SZ
@@ -234,6 +237,21 @@ def leap_scatter_turn_advantages(N, seg_offsets, seg_rollout, seg_turn, turn_adv
                                             _ptr(L), _ptr(totals), agg, _ptr(adv), _ptr(w), _stream(stream))
     _check(st, "leap_scatter_turn_advantages")
     return adv, w
+
+
+def leap_token_advantages(N, seg_offsets, seg_rollout, seg_turn, turn_adv, T_eff, *, M,
+                          agg=LEAP_AGG_SEQ_MEAN_TOKEN_MEAN, L=None, totals=None, adv=None, w=None, stream=None):
+    """Counts and scatter with the local totals in one call.  Returns (L, totals, adv, w)."""
+    n = T_eff.numel()
+    L = _empty(n, torch.int32, T_eff) if L is None else L
+    totals = _empty(2, torch.int64, T_eff) if totals is None else totals
+    adv = _empty(int(N), torch.float32, turn_adv) if adv is None else adv
+    w = _empty(int(N), torch.float32, turn_adv) if w is None else w
+    st = lib().leap_token_advantages(int(N), n, M, _ptr(seg_offsets), _ptr(seg_rollout), _ptr(seg_turn),
+                                     seg_rollout.numel(), _ptr(turn_adv), _ptr(T_eff), agg, _ptr(L), _ptr(totals),
+                                     _ptr(adv), _ptr(w), _stream(stream))
+    _check(st, "leap_token_advantages")
+    return L, totals, adv, w
 
 
 def _logits_args(logits, V):

@@ -6,6 +6,7 @@ stream:
   2. leap_rollout_token_counts     per-rollout optimised-token counts, local totals
   3. (data parallel) all_reduce(totals)  the one exchange: global loss normalisers
   4. leap_scatter_turn_advantages  per-token advantage and aggregation weight
+     (one process: steps 2 and 4 as one call, leap_token_advantages)
   5. leap_grpo_loss_fwd            clipped surrogate + fused dlogits (Eq. 3)
 Only step 3 leaves libleap, and only when a process group with more than one
 rank is passed in.  run() takes resident logits, run_chunked() a stream that
@@ -62,15 +63,19 @@ class GrpoStep:
         L.leap_group_rank_advantages(self.pass_turn, self.num_turns, G=b.G, M=b.M, tau_min=self.tau[0],
                                      tau_max=self.tau[1], gamma=self.gamma, eps_std=self.eps_std,
                                      gate_in=self.gate_in, out=self.rank_out)
+        if pg is None or torch.distributed.get_world_size(pg) == 1:   # counts + scatter in one launch
+            L.leap_token_advantages(b.N, self.seg_offsets, self.seg_rollout, self.seg_turn, self.rank_out["turn_adv"],
+                                    self.rank_out["T_eff"], M=b.M, agg=self.agg, L=self.L, totals=self.totals,
+                                    adv=self.adv, w=self.w)
+            return
         L.leap_rollout_token_counts(b.N, self.seg_offsets, self.seg_rollout, self.seg_turn,
                                     self.rank_out["T_eff"], M=b.M, L=self.L, totals=self.totals)
-        if pg is not None and torch.distributed.get_world_size(pg) > 1:
-            if torch.distributed.get_backend(pg) == "nccl":
-                torch.distributed.all_reduce(self.totals, group=pg)
-            else:   # a host backend (gloo): the two counters travel through host memory
-                host = self.totals.cpu()
-                torch.distributed.all_reduce(host, group=pg)
-                self.totals.copy_(host)
+        if torch.distributed.get_backend(pg) == "nccl":
+            torch.distributed.all_reduce(self.totals, group=pg)
+        else:   # a host backend (gloo): the two counters travel through host memory
+            host = self.totals.cpu()
+            torch.distributed.all_reduce(host, group=pg)
+            self.totals.copy_(host)
         L.leap_scatter_turn_advantages(b.N, self.seg_offsets, self.seg_rollout, self.seg_turn,
                                        self.rank_out["turn_adv"], self.rank_out["T_eff"], self.L, self.totals,
                                        M=b.M, agg=self.agg, adv=self.adv, w=self.w)
@@ -182,10 +187,20 @@ class GrpoStep:
             self._stage_key = key
         return self._stage
 
-    # libleap counts tokens in one launch up to this many rollouts, three above it.
+    # libleap counts tokens in one launch up to this many rollouts, three above it;
+    # counts and scatter share one launch for tables of up to 768 segments.
     ONE_BLOCK_COUNT_ROLLOUTS = 12000
+    ONE_LAUNCH_TOKEN_SEGMENTS = 768
 
-    def launches_per_run(self):
-        """Kernel launches one run() makes: rank 1, counts 1 (or 3), scatter 1, loss 1 + reduce 2."""
-        counts = 1 if self.b.n <= self.ONE_BLOCK_COUNT_ROLLOUTS else 3
-        return 1 + counts + 1 + 1 + 2
+    def token_launches(self, pg=None):
+        """Launches of steps 2-4: 1 when counts and scatter share a launch."""
+        b = self.b
+        single = pg is None or torch.distributed.get_world_size(pg) == 1
+        S = len(b.seg_rollout)
+        if single and S <= self.ONE_LAUNCH_TOKEN_SEGMENTS and 4 * b.n + 4 * (S + 1) + 12 * S <= 48 * 1024:
+            return 1
+        return (1 if b.n <= self.ONE_BLOCK_COUNT_ROLLOUTS else 3) + 1
+
+    def launches_per_run(self, pg=None):
+        """Kernel launches one run() makes: rank 1, tokens 1-4, loss 1 + reduce 2."""
+        return 1 + self.token_launches(pg) + 1 + 2

@@ -273,3 +273,40 @@ def test_lexi_special_keys(G):
     orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, 0, G, 0.8, cmp=O.CMP_LEXI,
                             speedup=sp.reshape(-1, G), ntokens=tok.reshape(-1, G))
     _compare(gpu, orc, M)
+
+
+@pytest.mark.parametrize("M", [1, 3, 8])
+def test_quad_pair_and_generic_kernels_agree_at_64(M):
+    """G = 64 runs the quad kernel (two groups per warp, 16-byte stores) when
+    the buffers allow it; outputs offset by 8 bytes send the call to the pair
+    kernel, by 4 bytes to the generic one.  An odd group count leaves the last
+    warp with one group.  All three equal the oracle and each other, bit for bit."""
+    G = 64
+    rng = np.random.default_rng(11 * M)
+    groups = 37
+    n = groups * G
+    nt = rng.integers(1, M + 1, size=n).astype(np.int8)
+    pt = np.minimum(np.where(rng.random(n) < 0.5, rng.integers(1, M + 1, size=n), 0), nt).astype(np.int8)
+    pt[70] = M + 1                                  # one malformed outcome
+    L = leap()
+    dev = torch.device("cuda")
+    pt_d, nt_d = torch.as_tensor(pt, device=dev), torch.as_tensor(nt, device=dev)
+    tau = (16, 48)
+    L.leap_get_device_status()
+    quad = L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=tau[0], tau_max=tau[1], gamma=0.8)
+    results = [quad]
+    for shift4, shift1 in ((2, 2), (1, 1)):         # 8-byte / 2-byte offsets (pair); 4-byte / 1-byte (generic)
+        off = lambda k, dt, sh: torch.empty(k + sh, dtype=dt, device=dev)[sh:]
+        out = dict(gate=off(groups, torch.uint8, shift1), r=off(n, torch.uint8, shift1),
+                   n_worse=off(n, torch.int32, shift4), n_better=off(n, torch.int32, shift4),
+                   R=off(n, torch.float32, shift4), A=off(n, torch.float32, shift4),
+                   turn_adv=off(n * M, torch.float32, shift4), T_eff=off(n, torch.uint8, shift1))
+        results.append(L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=tau[0], tau_max=tau[1],
+                                                    gamma=0.8, out=out))
+    torch.cuda.synchronize()
+    assert L.leap_get_device_status() & L.LEAP_DEV_BAD_OUTCOME
+    for other in results[1:]:
+        for k in quad:
+            assert torch.equal(quad[k], other[k]), k
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, tau[0], tau[1], 0.8)
+    _compare(quad, orc, M)
