@@ -40,9 +40,9 @@ WORKLOAD = ("single-turn GRPO: 16 prompts x G=8 x 256 token slots = 32,768 rows 
 # dram bytes (read + write) of one fused_loss_l2_kernel launch on this workload: an ncu capture of the
 # kernel built from sources with this SHA-256 on a 4,096-row slice, scaled to the full launch by
 # algorithmic bytes (traffic grows in proportion to them); null once the sources change.
-KNOWN_TRAFFIC = {"src_sha256": "485457ae5bfd97e4b93d539a63292f777878268f78af4bab4630090ffd84ec94", "bytes_per_launch": 16305801239}
+KNOWN_TRAFFIC = {"src_sha256": "fb8553ff1dfb58974c70d606b3c58638d05a8649102453714ff7f24d996d3702", "bytes_per_launch": 16264158836}
 KERNEL_SOURCES = ("paper_2608_01804_gb300/csrc/logprob_loss.cu", "paper_2608_01804_gb300/csrc/leap_common.cuh",
-                  "paper_2608_01804_gb300/csrc/loss_math.cuh")
+                  "paper_2608_01804_gb300/csrc/loss_math.cuh", "paper_2608_01804_gb300/csrc/row_math.cuh")
 
 
 def _src_sha():
@@ -70,6 +70,8 @@ def parse_args():
                     help="run only the rank advantages on 65,536 groups x 64 rollouts (M = 3), for profiling captures")
     ap.add_argument("--tokens-only", action="store_true",
                     help="run only the token counts + scatter on the packed multi-turn batch, for profiling captures")
+    ap.add_argument("--tokens-layout", choices=["multiturn", "tiny"], default="multiturn",
+                    help="with --tokens-only: the packed multi-turn batch or the small padded one")
     ap.add_argument("--logprobs-only", action="store_true",
                     help="run only the log-probs and the forward-only loss on the single-turn batch, for profiling")
     ap.add_argument("--short-rows", action="store_true",
@@ -682,18 +684,20 @@ def rank_only(args):
 
 
 def tokens_only(args):
-    """Per-rollout token counts + per-token scatter alone on the packed
-    multi-turn batch: --warmup untimed calls, then --steps timed ones, each
-    after an L2 flush; prints one JSON line."""
+    """Per-rollout token counts + per-token scatter alone (the two calls, then
+    the one-launch call) on the packed multi-turn batch or, with
+    --tokens-layout tiny, the small padded batch: --warmup untimed calls, then
+    --steps timed ones, each after an L2 flush; prints one JSON line."""
     from paper_2608_01804_gb300 import build
     build.build()
     from paper_2608_01804_gb300 import leap as L
     from paper_2608_01804_gb300 import synth
     device = torch.device("cuda", 0)
-    b = synth.multiturn_dcp_batch()
+    b = synth.tiny_batch() if args.tokens_layout == "tiny" else synth.multiturn_dcp_batch()
     pt_d = torch.as_tensor(b.pass_turn).to(device)
     nt_d = torch.as_tensor(b.num_turns).to(device)
-    rk = L.leap_group_rank_advantages(pt_d, nt_d, G=b.G, M=b.M, tau_min=8, tau_max=15, gamma=0.9)
+    tau = (0, b.G) if args.tokens_layout == "tiny" else (8, 15)
+    rk = L.leap_group_rank_advantages(pt_d, nt_d, G=b.G, M=b.M, tau_min=tau[0], tau_max=tau[1], gamma=0.9)
     so = torch.as_tensor(b.seg_offsets).to(device)
     sr = torch.as_tensor(b.seg_rollout).to(device)
     st_ = torch.as_tensor(b.seg_turn).to(device)

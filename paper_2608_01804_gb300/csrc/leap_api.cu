@@ -15,9 +15,6 @@ __device__ unsigned int g_leap_status;
 namespace {
 
 constexpr int kMaxDevices = 64;
-// The widest row the short-row kernel holds in the registers of one row group
-// (8 warps x 4 16-byte vectors of bf16 per thread).
-constexpr int64_t kShortRowV = 8192;
 
 std::mutex g_mu;
 unsigned int* g_status_ptr[kMaxDevices] = {};
@@ -291,12 +288,11 @@ leap_status_t leap_grpo_loss_fwd(const leap_loss_params_t* p, const uint16_t* lo
     if (dlogits && !aligned16(dlogits)) return LEAP_ERR_INVALID_ARG;
     if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return LEAP_ERR_INVALID_ARG;
     if (ws_bytes < loss_workspace_bytes(N)) return LEAP_ERR_INVALID_ARG;
-    // Rows of at most kShortRowV columns fit the registers of one row group,
-    // so the short-row kernel takes them whatever the flag: it holds each row
-    // on chip and reduces it with warp shuffles, where the persistent
-    // two-pass kernel's 1,024-thread CTAs would spend most of a short row in
-    // its block reductions.
-    const bool single_read = (p->flags & LEAP_LOSS_SINGLE_READ) != 0 || (int64_t)V <= kShortRowV;
+    // Rows of at most kShortRowMaxV columns take the short-row kernel whatever
+    // the flag (a group of warps holds each row on chip, read once), where the
+    // persistent two-pass kernel's 1,024-thread CTAs would spend most of a
+    // short row in its block reductions.
+    const bool single_read = (p->flags & LEAP_LOSS_SINGLE_READ) != 0 || V <= kShortRowMaxV;
     if (dlogits && single_read && (int64_t)V > fused_max_vocab()) return LEAP_ERR_UNSUPPORTED;
     const LossWorkspace ws = carve_loss_workspace(workspace, N);
     RowArgs a = {};

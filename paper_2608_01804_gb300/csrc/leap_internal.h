@@ -99,6 +99,9 @@ cudaError_t launch_row_stream(const RowArgs& a, int mode, cudaStream_t s);
 // cluster-resident one (cudaErrorNotSupported if V is too large for it).
 cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s);
 cudaError_t launch_split_bwd(const RowArgs& a, cudaStream_t s);
+// Fused forward + backward for rows of V <= kShortRowMaxV (short_rows.cu).
+constexpr int32_t kShortRowMaxV = 8192;
+cudaError_t launch_short_row_loss(const RowArgs& a, cudaStream_t s);
 cudaError_t launch_loss_reduce(const LossWorkspace& ws, int64_t N, float* loss, void* stats,
                                bool accumulate, cudaStream_t s);
 int64_t fused_max_vocab();

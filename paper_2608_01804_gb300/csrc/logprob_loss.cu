@@ -17,16 +17,14 @@
 //                      exchange one (max, sum) pair through distributed
 //                      shared memory: each row is read from HBM exactly once
 //                      whatever else uses L2 (LEAP_LOSS_SINGLE_READ).
-//   short_row_kernel   forward + backward for V <= 8,192: a group of 1-8
-//                      warps holds one row in registers (read once) and
-//                      reduces it with warp shuffles; persistent groups load
-//                      the next row while they write the current one.
+//   (rows of V <= 8,192 take short_row_kernel in short_rows.cu)
 //   split_bwd_kernel   dlogits from a saved lse: 2V read + 2V written.
 //   reduce kernels     fixed-order fp64 sum of the per-row loss terms.
 #include "../../include/leap.h"
 #include "leap_common.cuh"
 #include "leap_internal.h"
 #include "loss_math.cuh"
+#include "row_math.cuh"
 
 #include <algorithm>
 #include <math.h>
@@ -34,90 +32,6 @@
 
 namespace leap {
 namespace {
-
-__device__ __forceinline__ uint4 neg_inf4() {
-    return make_uint4(kNegInfBf16x2, kNegInfBf16x2, kNegInfBf16x2, kNegInfBf16x2);
-}
-
-// Sets elements n..7 of an 8 x bf16 vector to -inf (row tail beyond V).
-__device__ __forceinline__ void mask_tail(uint4& x, int n) {
-    uint32_t w[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        if (j >= n) {
-            if (j & 1) w[j >> 1] = (w[j >> 1] & 0x0000ffffu) | 0xff800000u;
-            else       w[j >> 1] = (w[j >> 1] & 0xffff0000u) | 0x0000ff80u;
-        }
-    }
-    x = make_uint4(w[0], w[1], w[2], w[3]);
-}
-
-// Stores vector vi of a dlogits row; the row's last vector keeps columns >= V intact.
-__device__ __forceinline__ void store_vec(uint4* drow, int64_t vi, uint4 val, int64_t V8, int tailn) {
-    if (tailn == 0 || vi != V8 - 1) {
-        st_stream(drow + vi, val);
-    } else {
-        uint16_t* p = reinterpret_cast<uint16_t*>(drow + vi);
-        const uint32_t w[4] = {val.x, val.y, val.z, val.w};
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-            if (j < tailn) p[j] = (uint16_t)((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xffffu));
-    }
-}
-
-__device__ __forceinline__ float bf16_at(const uint16_t* p) {
-    return __uint_as_float(((uint32_t)*p) << 16);
-}
-
-// Max of NV vectors of 8 bf16 as a balanced tree of packed maxima (depth
-// 2 + log2 NV instead of a 4 NV-long chain).
-template <int NV>
-__device__ __forceinline__ float tree_max(const uint4 (&x)[NV]) {
-    uint32_t v[NV];
-#pragma unroll
-    for (int k = 0; k < NV; ++k) v[k] = max_bf16x2(max_bf16x2(x[k].x, x[k].y), max_bf16x2(x[k].z, x[k].w));
-#pragma unroll
-    for (int stride = 1; stride < NV; stride *= 2) {
-#pragma unroll
-        for (int k = 0; k + stride < NV; k += 2 * stride) v[k] = max_bf16x2(v[k], v[k + stride]);
-    }
-    return fmaxf(bf16_lo(v[0]), bf16_hi(v[0]));
-}
-
-// Sum over NV vectors of 2^(z * c1 - mc), one accumulator per element
-// position (8 independent chains of length NV), then a tree.
-template <int NV>
-__device__ __forceinline__ float tree_exp_sum(const uint4 (&x)[NV], float c1, float mc) {
-    float acc[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) acc[j] = 0.f;
-#pragma unroll
-    for (int k = 0; k < NV; ++k) {
-        const uint32_t w[4] = {x[k].x, x[k].y, x[k].z, x[k].w};
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            acc[2 * q] += ex2(fmaf(bf16_lo(w[q]), c1, -mc));
-            acc[2 * q + 1] += ex2(fmaf(bf16_hi(w[q]), c1, -mc));
-        }
-    }
-    return ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
-}
-
-// dlogits of one vector: coef * (1[v = y] - 2^(z c1 - K)); `yl` is the target's
-// lane in this vector or -1.
-__device__ __forceinline__ uint4 dlogit8(const uint4& x, float c1, float K, float coef, int yl) {
-    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
-    uint32_t o[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        float lo = -coef * ex2(fmaf(bf16_lo(w[q]), c1, -K));
-        float hi = -coef * ex2(fmaf(bf16_hi(w[q]), c1, -K));
-        if (yl == 2 * q) lo += coef;
-        if (yl == 2 * q + 1) hi += coef;
-        o[q] = pack_bf16x2(lo, hi);
-    }
-    return make_uint4(o[0], o[1], o[2], o[3]);
-}
 
 // ---------------------------------------------------------------------------
 // Streaming single pass.  TPR threads per row (32: several rows per CTA;
@@ -523,278 +437,6 @@ __global__ void __launch_bounds__(T, 1) fused_loss_l2_kernel(RowArgs a) {
 }
 
 // ---------------------------------------------------------------------------
-// Fused forward + backward for short rows (V <= 8,192).  A row group of W
-// warps owns one row at a time; warp w of the group owns the contiguous slice
-// of 16-byte vectors [128 w, 128 (w + 1)) of the row (2 KB), lane l vectors
-// 128 w + l + 32 k (k < 4), so the row is read from HBM once.
-//   * Staging: each warp double-buffers its slice in shared memory.  While it
-//     works on row i, a 1-D bulk copy (TMA) of its slice of row i + 1 is in
-//     flight into the other stage, completing on that stage's mbarrier; every
-//     wait is bounded (LEAP_DEV_TIMEOUT).  Registers hold one row only.
-//   * Arithmetic: the kernel would otherwise be bound by instruction issue,
-//     so the row max is reduced first (packed bf16 maxima, then the warp), the
-//     exponentials 2^((z - m) c1) are taken once and kept in registers
-//     (32 fp32 per lane), element pairs go through packed fp32x2 FMA / add /
-//     multiply, and dlogits is one multiply per element.
-//   * W > 1: each warp publishes (max, sum) and, if it holds it, the target
-//     logit in shared memory behind one named barrier per live row (two
-//     alternating slots); every warp then merges the W pairs directly.
-//   * FULL (V a multiple of 1,024): every slice is whole, so the per-vector
-//     bounds and tail checks are compiled out.
-// Row groups are persistent and walk rows g, g + stride, ...  Masked rows are
-// not read.
-// ---------------------------------------------------------------------------
-constexpr int kShortThreads = 256;        // 8 warps per CTA
-constexpr int kShortNV = 4;               // 16-byte vectors per lane and row
-constexpr int kShortVPW = 32 * kShortNV;  // vectors per warp slice (2 KB)
-constexpr int kShortMinBlocks = 3;        // register budget: 80 per thread
-
-struct ShortSmem {
-    uint4 stage[kShortThreads / 32][2][kShortVPW];   // 32 KB: two 2 KB stages per warp
-    uint64_t full[kShortThreads / 32][2];            // one mbarrier per stage
-    float4 part[2][kShortThreads / 32];              // (max, sum, target logit, holds target) per warp
-    int abort_flag;
-};
-
-// Packed pairs of fp32 (Blackwell's f32x2 FMA / add / multiply: one
-// instruction for two lanes of arithmetic).
-__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
-    uint64_t r;
-    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
-    return r;
-}
-__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
-    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-}
-__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
-    uint64_t r;
-    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
-    return r;
-}
-__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
-    uint64_t r;
-    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-    return r;
-}
-__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
-    uint64_t r;
-    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-    return r;
-}
-
-template <int W, bool FULL>
-__global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kernel(RowArgs a) {
-    constexpr int NV = kShortNV, VPW = kShortVPW, TG = 32 * W, GPB = kShortThreads / TG;
-    __shared__ __align__(128) ShortSmem sm;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int gib = warp / W;                  // row group within the block
-    const int wig = warp % W;                  // warp within the row group
-    // 32-bit row and vector indices (N < 2^31 is checked on the host; V8 <= 1,024).
-    const int stride = (int)gridDim.x * GPB;
-    const int N = (int)a.N;
-    const int V = a.V;
-    const int V8 = FULL ? W * VPW : (V + 7) >> 3;
-    const int tailn = FULL ? 0 : (V & 7);
-    const float c1 = a.inv_temp * kLog2e;
-    const int vbase = wig * VPW;                                  // this warp's first vector
-    const int nvec = FULL ? VPW : max(0, min(VPW, V8 - vbase));   // vectors in this warp's slice
-    const uint32_t slice_bytes = (uint32_t)nvec * 16u;
-
-    if (threadIdx.x == 0) sm.abort_flag = 0;
-    if (lane == 0) {
-        mbar_init(&sm.full[warp][0], 1);
-        mbar_init(&sm.full[warp][1], 1);
-        fence_mbar_init();
-    }
-    __syncthreads();
-
-    auto is_live = [&](float wr, int idr) { return wr != 0.f && idr >= 0 && idr < V; };
-    uint32_t phase = 0;     // bit s: parity of the next completion of stage s
-    uint32_t pending = 0;   // bit s: a copy into stage s has not been waited for
-    // Lane 0 starts the copy of this warp's slice of row r into stage st (none
-    // once a wait of this CTA has given up, so at most one copy per stage is
-    // ever outstanding).
-    auto issue = [&](int r, int st) {
-        if (slice_bytes == 0 || *reinterpret_cast<volatile int*>(&sm.abort_flag)) return;
-        pending |= 1u << st;
-        if (lane == 0) {
-            mbar_arrive_expect_tx(&sm.full[warp][st], slice_bytes);
-            bulk_g2s(&sm.stage[warp][st][0], a.logits + (int64_t)r * a.ld + (int64_t)vbase * 8, slice_bytes,
-                     &sm.full[warp][st]);
-        }
-    };
-    // w and id of the row `k` strides after `r`, or (0, 0) past the end.
-    auto scalars = [&](int r, int k, float& wr, int& idr) {
-        wr = 0.f;
-        idr = 0;
-        if (r < N - k * stride) {   // r + k * stride < N without overflow
-            wr = a.w[r + k * stride];
-            idr = a.ids[r + k * stride];
-        }
-    };
-
-    int row = (int)blockIdx.x * GPB + gib;
-    float w0, w1, w2;
-    int id0, id1, id2;
-    scalars(row, 0, w0, id0);
-    scalars(row, 1, w1, id1);
-    scalars(row, 2, w2, id2);
-    if (row < N && is_live(w0, id0)) issue(row, 0);
-    if (is_live(w1, id1)) issue(row + stride, 1);
-    int par = 0;
-    const uint64_t c1x2 = f2_pack(c1, c1);
-
-    for (int it = 0; row < N; row += stride, ++it) {
-        const int st = it & 1;
-        float w3;
-        int id3;
-        scalars(row, 3, w3, id3);
-
-        const bool bad = (w0 != 0.f) && (id0 < 0 || id0 >= V);
-        uint4* drow = reinterpret_cast<uint4*>(a.dlogits + (int64_t)row * a.ld);
-        if (w0 == 0.f || bad) {   // masked row: the same branch in every warp of the group
-#pragma unroll
-            for (int k = 0; k < NV; ++k) {
-                const int vi = vbase + lane + 32 * k;
-                if (FULL || vi < V8) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
-            }
-            if (wig == 0 && lane == 0) {
-                write_masked_outputs(a, row);
-                if (bad) flag_status(a.status, LEAP_DEV_BAD_ID);
-            }
-            if (is_live(w2, id2)) issue(row + 2 * stride, st);   // this row left stage st unused
-        } else {
-            const float old = a.old_logp[row], A = a.adv[row];
-            uint4 x[NV];
-            if (pending & (1u << st)) {
-                if (mbar_wait(&sm.full[warp][st], (phase >> st) & 1u, a.status, &sm.abort_flag)) {
-                    phase ^= 1u << st;
-                    pending &= ~(1u << st);
-                }   // else: results undefined (LEAP_DEV_TIMEOUT); the copy stays pending
-            }
-#pragma unroll
-            for (int k = 0; k < NV; ++k) {
-                const int li = lane + 32 * k;
-                if (FULL) {
-                    x[k] = sm.stage[warp][st][li];
-                } else {
-                    x[k] = (li < nvec) ? sm.stage[warp][st][li] : neg_inf4();
-                    if (tailn && vbase + li == V8 - 1) mask_tail(x[k], tailn);
-                }
-            }
-            // The target logit, if it lies in this warp's slice.
-            const int yl = id0 - vbase * 8;
-            const bool own_y = yl >= 0 && yl < nvec * 8;
-            float zy = own_y ? bf16_at(reinterpret_cast<const uint16_t*>(&sm.stage[warp][st][0]) + yl) : 0.f;
-            // Every lane has read the stage: it may take the copy of row i + 2.
-            __syncwarp();
-            fence_proxy_async_smem();
-            if (is_live(w2, id2)) issue(row + 2 * stride, st);
-            // Row max: packed maxima, then the warp.
-            float m = tree_max(x);
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-            // Exponentials against the warp max, kept (as pairs) for the backward.
-            uint64_t e2[NV][4];
-            float ssum = 0.f;
-            if (m != -INFINITY) {
-                const float nmc = -m * c1;
-                const uint64_t nmc2 = f2_pack(nmc, nmc);
-                uint64_t acc2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
-#pragma unroll
-                for (int k = 0; k < NV; ++k) {
-                    const uint32_t wv[4] = {x[k].x, x[k].y, x[k].z, x[k].w};
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        float lo, hi;
-                        f2_unpack(f2_fma(f2_pack(bf16_lo(wv[q]), bf16_hi(wv[q])), c1x2, nmc2), lo, hi);
-                        e2[k][q] = f2_pack(ex2(lo), ex2(hi));
-                        acc2[q & 1] = f2_add(acc2[q & 1], e2[k][q]);
-                    }
-                }
-                float s0, s1, s2, s3;
-                f2_unpack(acc2[0], s0, s1);
-                f2_unpack(acc2[1], s2, s3);
-                ssum = (s0 + s1) + (s2 + s3);
-            } else {
-#pragma unroll
-                for (int k = 0; k < NV; ++k)
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) e2[k][q] = f2_pack(0.f, 0.f);
-            }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) ssum += __shfl_xor_sync(0xffffffffu, ssum, o);
-            // The row's (max, sum), the target logit and this warp's factor 2^((m_warp - m_row) c1).
-            float mrow = m, srow = ssum, wscale = 1.f;
-            if (W > 1) {
-                if (lane == 0) sm.part[par][warp] = make_float4(m, ssum, zy, own_y ? 1.f : 0.f);
-                named_bar_sync(1 + gib, TG);
-                float4 p[W];
-#pragma unroll
-                for (int v = 0; v < W; ++v) p[v] = sm.part[par][gib * W + v];
-                mrow = p[0].x;
-#pragma unroll
-                for (int v = 1; v < W; ++v) mrow = fmaxf(mrow, p[v].x);
-                srow = 0.f;
-#pragma unroll
-                for (int v = 0; v < W; ++v) {
-                    if (p[v].y != 0.f) srow = fmaf(p[v].y, ex2((p[v].x - mrow) * c1), srow);
-                    if (p[v].w != 0.f) zy = p[v].z;
-                }
-                wscale = (ssum != 0.f) ? ex2((m - mrow) * c1) : 0.f;
-                par ^= 1;   // live rows alternate slots: a slot is rewritten only after the
-                            // next live row's barrier, which every reader of it has passed
-            }
-            const TokenLoss r = token_loss(a, mrow, srow, zy, old, A, w0);
-            const float coef = a.grad_scale * r.g * a.inv_temp;
-            if (wig == 0 && lane == 0) write_row_outputs(a, row, r, w0);
-            // dlogits_v = coef (1[v = y] - e_v wscale / s_row); the factor's own
-            // rounding (fast reciprocal, ~2 ulp of fp32) is far below bf16's.
-            const float nf = -__fdividef(coef * wscale, srow);
-            const uint64_t nf2 = f2_pack(nf, nf);
-            const int yv = id0 >> 3;
-            const int ylane = id0 & 7;
-#pragma unroll
-            for (int k = 0; k < NV; ++k) {
-                const int vi = vbase + lane + 32 * k;
-                if (FULL || vi < V8) {
-                    uint4 d = make_uint4(0, 0, 0, 0);
-                    if (coef != 0.f) {
-                        float o8[8];
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) f2_unpack(f2_mul(e2[k][q], nf2), o8[2 * q], o8[2 * q + 1]);
-                        if (vi == yv) {
-#pragma unroll
-                            for (int j = 0; j < 8; ++j)
-                                if (j == ylane) o8[j] += coef;
-                        }
-                        d = make_uint4(pack_bf16x2(o8[0], o8[1]), pack_bf16x2(o8[2], o8[3]),
-                                       pack_bf16x2(o8[4], o8[5]), pack_bf16x2(o8[6], o8[7]));
-                    }
-                    if (FULL) st_stream(drow + vi, d);
-                    else store_vec(drow, vi, d, V8, tailn);
-                }
-            }
-        }
-        // Shift the scalar pipeline by one row.
-        w0 = w1;
-        id0 = id1;
-        w1 = w2;
-        id1 = id2;
-        w2 = w3;
-        id2 = id3;
-    }
-    // Every copy is waited for before its row is used, so one can still be in
-    // flight here only after a wait gave up: wait for it (bounded again) so no
-    // copy lands in the shared memory of an exited CTA.
-    if (pending) {
-        volatile int fresh = 0;
-        for (int st = 0; st < 2; ++st)
-            if (pending & (1u << st)) mbar_wait(&sm.full[warp][st], (phase >> st) & 1u, a.status, &fresh);
-    }
-}
-
-// ---------------------------------------------------------------------------
 // Split backward from the saved lse.  Every thread recomputes the row's scalar
 // coefficient from broadcast loads, so no block synchronisation is needed.
 // ---------------------------------------------------------------------------
@@ -1053,48 +695,9 @@ cudaError_t launch_split_bwd(const RowArgs& a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-// Persistent grid of the short-row kernel: the CTAs that fit at once (cached
-// per device), at most one row group per row.
-template <int W, bool FULL>
-cudaError_t launch_short_rows(const RowArgs& a, cudaStream_t s) {
-    static std::mutex mu;
-    static int cached_dev = -1, cached_resident = 0;
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    int resident = 0;   // CTAs resident at once on the whole device
-    {
-        std::lock_guard<std::mutex> lk(mu);
-        if (cached_dev != dev) {
-            int per_sm = 0;
-            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, short_row_kernel<W, FULL>, kShortThreads, 0);
-            if (e != cudaSuccess) return e;
-            cached_dev = dev;
-            cached_resident = per_sm * device_sm_count();
-        }
-        resident = cached_resident;
-    }
-    if (resident <= 0) return cudaErrorNotSupported;
-    constexpr int GPB = kShortThreads / (32 * W);
-    const int64_t blocks = std::min<int64_t>((a.N + GPB - 1) / GPB, (int64_t)resident);
-    short_row_kernel<W, FULL><<<(unsigned)blocks, kShortThreads, 0, s>>>(a);
-    return cudaGetLastError();
-}
-
 cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s) {
     if (a.N == 0) return cudaSuccess;
-    const int64_t V8s = ((int64_t)a.V + 7) >> 3;
-    if (V8s <= (int64_t)8 * 32 * kShortNV) {   // V <= 8,192: the row lives in one row group's registers
-        const int W = V8s <= kShortVPW ? 1 : V8s <= 2 * kShortVPW ? 2 : V8s <= 4 * kShortVPW ? 4 : 8;
-        // Whole 2 KB slices for every warp (V = 1,024 W): no per-vector bounds checks.
-        const bool full = a.V == W * 8 * kShortVPW;
-        switch (W) {
-            case 1: return full ? launch_short_rows<1, true>(a, s) : launch_short_rows<1, false>(a, s);
-            case 2: return full ? launch_short_rows<2, true>(a, s) : launch_short_rows<2, false>(a, s);
-            case 4: return full ? launch_short_rows<4, true>(a, s) : launch_short_rows<4, false>(a, s);
-            default: return full ? launch_short_rows<8, true>(a, s) : launch_short_rows<8, false>(a, s);
-        }
-    }
+    if (a.V <= kShortRowMaxV) return launch_short_row_loss(a, s);   // short_rows.cu
     if (!single_read) {
         RowArgs b = a;
         const int64_t grid = std::min<int64_t>(a.N, (int64_t)device_sm_count());

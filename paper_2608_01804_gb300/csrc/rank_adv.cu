@@ -536,6 +536,7 @@ __global__ void __launch_bounds__(256, kQuadMinBlocks) rank_quad_kernel(RankArgs
     constexpr int J = 4, M = MC, G = 64;
     const int lane = threadIdx.x & 31;
     const int half = lane >> 4;
+
     const int64_t npairs = ((int64_t)a.num_groups + 1) / 2;
     const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
     for (int64_t pr = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); pr < npairs; pr += warps) {
@@ -717,13 +718,27 @@ __global__ void __launch_bounds__(kCountThreads) counts_one_block_kernel(SegArgs
     const int n = a.n_rollouts;
     for (int i = threadIdx.x; i < n; i += kCountThreads) sL[i] = 0;
     __syncthreads();
-    for (int64_t s = threadIdx.x; s < a.num_segs; s += kCountThreads) {
-        int32_t lo, hi, i, t;
-        if (!segment_ok(a, s, lo, hi, i, t)) {
-            flag_status(a.status, 4u);
-            continue;
+    // Two segments per thread per pass, both segments' fields and turn counts
+    // loaded before either is counted (two dependent load rounds per pass
+    // instead of four).
+    for (int64_t s0 = threadIdx.x; s0 < a.num_segs; s0 += 2 * kCountThreads) {
+        int32_t lo[2], hi[2], i[2], t[2];
+        bool ok[2], use[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int64_t s = s0 + (int64_t)u * kCountThreads;
+            ok[u] = s < a.num_segs && segment_ok(a, s, lo[u], hi[u], i[u], t[u]);
+            if (s < a.num_segs && !ok[u]) flag_status(a.status, 4u);
         }
-        if (t >= 0 && hi > lo && t < (int)a.T_eff[i]) atomicAdd(&sL[i], hi - lo);
+        int te[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            use[u] = ok[u] && t[u] >= 0 && hi[u] > lo[u];
+            te[u] = use[u] ? (int)a.T_eff[i[u]] : 0;
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u)
+            if (use[u] && t[u] < te[u]) atomicAdd(&sL[i[u]], hi[u] - lo[u]);
     }
     __syncthreads();
     long long tok = 0, roll = 0;
@@ -823,13 +838,19 @@ __global__ void __launch_bounds__(256) scatter_kernel(SegArgs a) {
         }
         int32_t cur = -1, clo = 0, chi = 0;
         float cadv = 0.f, cw = 0.f;
+        // Start of the segment after `seg` (kept in a register: reloaded only
+        // when the walk moves on).
+        int64_t nxt = (S > 0 && seg + 1 < S) ? (int64_t)a.seg_offsets[seg + 1] : INT64_MAX;
 #pragma unroll 1
         for (int it = 0; it < kScatterIters; ++it) {
             const int64_t k = k0 + it * 32 + lane;
             if (k >= a.N) break;
             float adv = 0.f, w = 0.f;
             if (S > 0) {
-                while (seg + 1 < S && a.seg_offsets[seg + 1] <= k) ++seg;
+                while (nxt <= k) {
+                    ++seg;
+                    nxt = (seg + 1 < S) ? (int64_t)a.seg_offsets[seg + 1] : INT64_MAX;
+                }
                 if (seg != cur) {   // entering a segment: its fields, advantage and weight
                     cur = seg;
                     int32_t i, t;
