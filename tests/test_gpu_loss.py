@@ -186,3 +186,33 @@ def test_empty_batch():
     loss = torch.full((1,), 5.0, device="cuda")
     L.leap_grpo_loss_fwd(z, ids, e, e, e, loss=loss)
     assert loss.item() == 0.0
+
+
+@pytest.mark.parametrize("N,pattern", [(1, "live"), (151, "random"), (152, "masked"), (153, "runs"),
+                                       (1000, "live"), (3001, "runs"), (3001, "random"), (5000, "head")])
+def test_two_pass_kernel_row_partition(N, pattern):
+    """The two-pass kernel's persistent CTAs share the rows out among
+    themselves: every row is written, whatever the pattern of live and masked
+    rows and whether N is below, at or above the CTA count, and the loss
+    equals the oracle's sum over all rows."""
+    L = leap()
+    L.leap_get_device_status()
+    V = 9000                                   # above the short-row limit: the two-pass kernel
+    z, ids, old, adv, w = _inputs(N, V, seed=N % 53 + 60, sigma=3.0, spikes=0.01, old_sigma=0.3, mask_frac=0.0)
+    r = np.arange(N)
+    keep = {"live": np.ones(N, bool), "masked": np.zeros(N, bool), "random": np.random.default_rng(N).random(N) < 0.6,
+            "runs": (r // 97) % 3 != 1, "head": r < N // 7}[pattern]
+    w.mul_(torch.as_tensor(keep.astype(np.float32), device="cuda"))
+    dl = torch.full_like(z, float("nan"))
+    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, dlogits=dl)
+    assert L.leap_get_device_status() == 0
+    assert not torch.isnan(dl).any()          # every row written
+    assert torch.all(dl[torch.as_tensor(~keep, device="cuda")] == 0)
+    rows = list(range(N))
+    orc = _oracle_rows(z, ids, old, adv, w, rows, V)
+    if keep.any():
+        assert abs(out["loss"].item() - orc["loss"]) <= TOL_LOSS_REL * abs(orc["loss"])
+    else:
+        assert out["loss"].item() == 0.0
+    sample = sorted(set(np.linspace(0, N - 1, min(N, 48)).astype(int).tolist()))
+    _check_rows(out, _oracle_rows(z, ids, old, adv, w, sample, V), sample, V, dl=dl)
