@@ -123,6 +123,80 @@ def measured_peaks():
     return 6800.0, "fallback"
 
 
+class NvmlClockSampler:
+    """Samples of this GPU's SM clock, power and clock-event reasons every
+    `interval` seconds from a host thread through NVML (libnvidia-ml, read-only
+    queries), so that even a timed region of a few tens of milliseconds gets
+    several samples.  Raises OSError where NVML cannot be loaded."""
+
+    REASONS = ((0x8, "hw_slowdown"), (0x40, "hw_thermal_slowdown"), (0x20, "sw_thermal_slowdown"),
+               (0x4, "sw_power_cap"), (0x80, "hw_power_brake_slowdown"))
+
+    def __init__(self, device, interval=0.005):
+        import ctypes
+        import threading
+        self.ct = ctypes
+        self.threading = threading
+        self.nvml = ctypes.CDLL("libnvidia-ml.so.1")
+        if self.nvml.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit failed")
+        uuid = str(torch.cuda.get_device_properties(device).uuid)
+        if not uuid.startswith("GPU-"):
+            uuid = "GPU-" + uuid
+        self.h = ctypes.c_void_p()
+        if self.nvml.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(self.h)) != 0:
+            raise OSError("no NVML handle for " + uuid)
+        self.reasons_fn = getattr(self.nvml, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            getattr(self.nvml, "nvmlDeviceGetCurrentClocksThrottleReasons")
+        self.interval = interval
+        self.samples = []
+        self.stop_evt = threading.Event()
+        self.thread = None
+        self.max_mhz = self._uint(self.nvml.nvmlDeviceGetMaxClockInfo, 1)
+
+    def _uint(self, fn, *args):
+        v = self.ct.c_uint(0)
+        return v.value if fn(self.h, *args, self.ct.byref(v)) == 0 else None
+
+    def _sample(self):
+        sm = self._uint(self.nvml.nvmlDeviceGetClockInfo, 1)
+        mw = self._uint(self.nvml.nvmlDeviceGetPowerUsage)
+        r = self.ct.c_ulonglong(0)
+        reasons = r.value if self.reasons_fn(self.h, self.ct.byref(r)) == 0 else 0
+        if sm is not None:
+            self.samples.append((sm, mw, reasons))
+
+    def _run(self):
+        while not self.stop_evt.is_set():
+            self._sample()
+            self.stop_evt.wait(self.interval)
+
+    def start(self):
+        self.samples = []
+        self.stop_evt.clear()
+        self.thread = self.threading.Thread(target=self._run, daemon=True)
+        self.thread.start()
+
+    def stop(self):
+        self.stop_evt.set()
+        self.thread.join()
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": ["no samples"], "source": "nvml"}
+        reasons = sorted({nm for _, _, bits in self.samples for b, nm in self.REASONS if bits & b})
+        power = [mw / 1000.0 for _, mw, _ in self.samples if mw is not None]
+        return {"sm_mhz": statistics.median(sm for sm, _, _ in self.samples), "sm_max_mhz": self.max_mhz,
+                "samples": len(self.samples), "power_w_max": max(power) if power else None, "reasons": reasons,
+                "source": "nvml, %g ms interval" % (1000 * self.interval)}
+
+
+def clock_sampler(device):
+    """NVML sampling where the library loads, else nvidia-smi."""
+    try:
+        return NvmlClockSampler(device)
+    except (OSError, AttributeError):
+        return ClockSampler(device)
+
+
 class ClockSampler:
     """nvidia-smi samples of this GPU's clocks and throttle reasons every 200 ms."""
 
@@ -859,7 +933,7 @@ def main():
 
     K = args.steps
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    clocks = ClockSampler(device)
+    clocks = clock_sampler(device)
     barrier()
     torch.cuda.synchronize()
     clocks.start()

@@ -885,9 +885,12 @@ __global__ void __launch_bounds__(256) scatter_kernel(SegArgs a) {
 // segment its advantage, weight and the end of its weighted tokens; then its
 // warps scatter their 256-token chunks with the same 32-ary search and walk
 // as scatter_kernel, reading the segment table from shared memory instead of
-// chasing dependent global loads.  Block 0 also writes L and the totals.  The
-// counting is repeated by every block (a few KB of the segment table read from
-// L2 per block) in exchange for one launch instead of two.
+// chasing dependent global loads.  The segment table (offsets, rollout, turn)
+// and T_eff are copied into shared memory in one round of independent loads,
+// so the counting needs no global load and the per-segment step one more round
+// (its turn advantage).  Block 0 also writes L and the totals.  The counting
+// is repeated by every block (a few KB of the segment table read from L2 per
+// block) in exchange for one launch instead of two.
 constexpr int kTokThreads = 256;
 // Every block repeats the table work, so the one launch pays off on small
 // tables only (measured: 117 / 255 segments 0.75 / 0.71 of the two launches'
@@ -895,7 +898,11 @@ constexpr int kTokThreads = 256;
 constexpr int kTokMaxSegs = 768;
 constexpr size_t kTokSmemMax = 48 * 1024;
 
-size_t fused_tok_smem(int64_t n, int64_t S) { return 4 * (size_t)n + 4 * ((size_t)S + 1) + 12 * (size_t)S; }
+// Shared memory of token_adv_fused_kernel: L and T_eff per rollout; offsets,
+// weighted end, advantage, weight, rollout and turn per segment.
+size_t fused_tok_smem(int64_t n, int64_t S) {
+    return 4 * (size_t)n + 4 * ((size_t)S + 1) + 17 * (size_t)S + (size_t)n + 16;
+}
 
 __global__ void __launch_bounds__(kTokThreads) token_adv_fused_kernel(SegArgs a) {
     extern __shared__ __align__(16) int32_t tsm[];
@@ -905,18 +912,30 @@ __global__ void __launch_bounds__(kTokThreads) token_adv_fused_kernel(SegArgs a)
     int32_t* send = soff + S + 1;                         // [S] end of the weighted tokens (= start if none)
     float* sadv = reinterpret_cast<float*>(send + S);     // [S]
     float* sw = sadv + S;                                 // [S]
+    int32_t* srol = reinterpret_cast<int32_t*>(sw + S);   // [S] seg_rollout
+    int8_t* sturn = reinterpret_cast<int8_t*>(srol + S);  // [S] seg_turn
+    uint8_t* ste = reinterpret_cast<uint8_t*>(sturn + S); // [n] T_eff
     __shared__ long long red[2][kTokThreads / 32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
-    for (int i = tid; i < n; i += kTokThreads) sL[i] = 0;
+    for (int i = tid; i < n; i += kTokThreads) {
+        sL[i] = 0;
+        ste[i] = a.T_eff[i];
+    }
     if (S > 0)
-        for (int q = tid; q <= S; q += kTokThreads) soff[q] = a.seg_offsets[q];
+        for (int q = tid; q <= S; q += kTokThreads) {
+            soff[q] = a.seg_offsets[q];
+            if (q < S) {
+                srol[q] = a.seg_rollout[q];
+                sturn[q] = a.seg_turn[q];
+            }
+        }
     __syncthreads();
     auto seg_fields = [&](int q, int& lo, int& hi, int& i, int& t) {
         lo = soff[q];
         hi = soff[q + 1];
-        t = a.seg_turn[q];
-        i = a.seg_rollout[q];
+        t = sturn[q];
+        i = srol[q];
         return lo >= 0 && hi >= lo && (int64_t)hi <= a.N && t < a.M && (t < 0 || (i >= 0 && i < n));
     };
     for (int q = tid; q < S; q += kTokThreads) {   // L_i (Sec. 3.3 token sets)
@@ -925,7 +944,7 @@ __global__ void __launch_bounds__(kTokThreads) token_adv_fused_kernel(SegArgs a)
             if (blockIdx.x == 0) flag_status(a.status, 4u);
             continue;
         }
-        if (t >= 0 && hi > lo && t < (int)a.T_eff[i]) atomicAdd(&sL[i], hi - lo);
+        if (t >= 0 && hi > lo && t < (int)ste[i]) atomicAdd(&sL[i], hi - lo);
     }
     __syncthreads();
     long long tok = 0, roll = 0;
@@ -960,7 +979,7 @@ __global__ void __launch_bounds__(kTokThreads) token_adv_fused_kernel(SegArgs a)
         const bool ok = seg_fields(q, lo, hi, i, t);
         float av = 0.f, wv = 0.f;
         int end = lo;
-        if (ok && t >= 0 && t < (int)a.T_eff[i]) {
+        if (ok && t >= 0 && t < (int)ste[i]) {
             av = a.turn_adv[(int64_t)i * a.M + t];
             if (a.agg == 1) {
                 wv = nv > 0 ? recip_count((double)nv) : 0.f;
