@@ -37,11 +37,11 @@ WORKLOAD = ("single-turn GRPO: 16 prompts x G=8 x 256 token slots = 32,768 rows 
             "rest masked padding), V=151936, bf16 logits N(0,3^2) + 1% spikes of +15, old log-probs = current "
             "+ N(0,0.05^2), clip eps 0.2/0.2, seq-mean-token-mean aggregation")
 
-# dram bytes (read + write) of one fused_loss_l2_kernel launch on this workload: an ncu capture of the
+# dram bytes (read + write) of one fused_loss_pipe_kernel launch on this workload: an ncu capture of the
 # kernel built from sources with this SHA-256 on a 4,096-row slice, scaled to the full launch by
 # algorithmic bytes (traffic grows in proportion to them); null once the sources change.
-KNOWN_TRAFFIC = {"src_sha256": "fb8553ff1dfb58974c70d606b3c58638d05a8649102453714ff7f24d996d3702", "bytes_per_launch": 16264158836}
-KERNEL_SOURCES = ("paper_2608_01804_gb300/csrc/logprob_loss.cu", "paper_2608_01804_gb300/csrc/leap_common.cuh",
+KNOWN_TRAFFIC = {"src_sha256": "a3375e545f1557fd1993cb6e7bbdb4f0506ad2c086270210ffca1e2b8f7bb7e6", "bytes_per_launch": 16223388660}
+KERNEL_SOURCES = ("paper_2608_01804_gb300/csrc/loss_pipe.cu", "paper_2608_01804_gb300/csrc/leap_common.cuh",
                   "paper_2608_01804_gb300/csrc/loss_math.cuh", "paper_2608_01804_gb300/csrc/row_math.cuh")
 
 
@@ -970,7 +970,7 @@ def main():
               "frac_of_nominal_7900_gbs": achieved / 7900.0}
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "launch_spread": spread,
-                "traffic": traffic, "kernel": "fused_loss_l2_kernel<1024,4,6> persistent (+2 reduce launches in the timing)",
+                "traffic": traffic, "kernel": "fused_loss_pipe_kernel<4,8,3,11,1024> persistent, rows pipelined (+2 reduce launches in the timing)",
                 "algorithmic_bytes_per_launch": alg_bytes, "launch_ms": loss_ms, "peak_source": peak_kind}
 
     # End to end through the same public calls, inputs copied from pinned host memory every step.

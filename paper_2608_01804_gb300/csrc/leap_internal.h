@@ -68,7 +68,6 @@ struct RowArgs {
     float* ws_rho;
     uint8_t* ws_flag;
     unsigned int* status;
-    int32_t next_stride;  // fused two-pass kernel: rows between a CTA's successive rows (its grid size)
 };
 
 // Workspace carve-up of leap_grpo_loss_fwd.
@@ -95,10 +94,14 @@ cudaError_t launch_token_advantages(const SegArgs& a, cudaStream_t s);
 
 // mode: 0 = log-probs only, 1 = loss forward (no dlogits).
 cudaError_t launch_row_stream(const RowArgs& a, int mode, cudaStream_t s);
-// Fused forward + backward: the L2 two-pass kernel, or with single_read the
-// cluster-resident one (cudaErrorNotSupported if V is too large for it).
+// Fused forward + backward: the row-pipelined two-pass kernel, or with
+// single_read the cluster-resident one (cudaErrorNotSupported if V is too
+// large for it).
 cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s);
 cudaError_t launch_split_bwd(const RowArgs& a, cudaStream_t s);
+// Fused forward + backward with the two passes of consecutive rows overlapped
+// on each SM through bulk-copy rings (loss_pipe.cu).
+cudaError_t launch_pipe_loss(const RowArgs& a, cudaStream_t s);
 // Fused forward + backward for rows of V <= kShortRowMaxV (short_rows.cu).
 constexpr int32_t kShortRowMaxV = 8192;
 cudaError_t launch_short_row_loss(const RowArgs& a, cudaStream_t s);

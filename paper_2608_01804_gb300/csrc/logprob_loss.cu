@@ -5,13 +5,8 @@
 //   row_stream_kernel  one pass over each logits row with an online
 //                      (max, sum) -> log-probs, or the loss forward without
 //                      dlogits.  2V bytes read per row.
-//   fused_loss_l2_kernel  forward + backward, one persistent CTA per SM taking
-//                      rows round-robin, two passes per row, the second
-//                      served by L2.  2V read + 2V written per row.  A bulk
-//                      L2 prefetch puts the whole row's HBM reads in flight
-//                      at once, and the head of the CTA's next row is
-//                      prefetched while this one writes, so reads and writes
-//                      overlap on every SM.
+//   (the default fused forward + backward is fused_loss_pipe_kernel in
+//   loss_pipe.cu: two passes per row, pipelined across rows on every SM)
 //   fused_loss_kernel  forward + backward with the row split over a cluster
 //                      of C CTAs that keep their slices in registers and
 //                      exchange one (max, sum) pair through distributed
@@ -303,140 +298,6 @@ __global__ void __launch_bounds__(T + 32, MINB) fused_loss_kernel(RowArgs a, int
 }
 
 // ---------------------------------------------------------------------------
-// Fused forward + backward (default): one persistent CTA of T threads per SM
-// taking rows round-robin, two passes over each row.  A bulk L2 prefetch puts
-// the whole row's reads in flight; the first pass reads it (evict_last) and
-// reduces it; the second reads it back (evict_first) and writes dlogits with
-// streaming stores, while the head of the CTA's next row is prefetched.  With
-// one row per SM in flight (152 rows, 46 MB at V = 151,936) the second read is
-// an L2 hit: DRAM sees 2V bytes read and 2V written per live row.
-// ---------------------------------------------------------------------------
-// Measured settings (the alternatives are in the kernel's profile summary):
-constexpr int kL2Threads = 1024;           // one CTA per SM (512 x 2 and 256 x 4 overflow L2)
-constexpr int kL2U1 = 4;                   // 16-byte vectors in flight per thread, pass 1 (2: 0.850, 8: 0.791)
-constexpr int kL2U2 = 6;                   // and pass 2 (2: 0.824, 4: 0.874, 5-8: 0.882-0.883, 10 spills)
-constexpr int64_t kPfChunk = 32768;        // bytes per bulk L2 prefetch request
-constexpr int64_t kNextBytes = 65536;      // head of the next row prefetched during pass 2
-// Warp-wide: bulk L2 prefetch of the first min(cap, row) bytes of a logits row.
-__device__ __forceinline__ void prefetch_row_l2(const uint16_t* zr, int V, int64_t cap, uint64_t policy, int lane) {
-    int64_t bytes = (int64_t)(V & ~7) * 2;
-    if (bytes > cap) bytes = cap & ~int64_t(15);
-    for (int64_t off = (int64_t)lane * kPfChunk; off < bytes; off += 32 * kPfChunk)
-        bulk_prefetch_l2(reinterpret_cast<const char*>(zr) + off,
-                         (uint32_t)(bytes - off < kPfChunk ? bytes - off : kPfChunk), policy);
-}
-// This CTA's next row (next_stride rows on), if it is live: prefetch its head
-// so that its pass 1 overlaps this row's writes.
-__device__ __forceinline__ void prefetch_next_row(const RowArgs& a, int64_t row, uint64_t policy, int lane) {
-    const int64_t nr = row + a.next_stride;
-    if (a.next_stride > 0 && nr < a.N && a.w[nr] != 0.f)
-        prefetch_row_l2(a.logits + nr * a.ld, a.V, kNextBytes, policy, lane);
-}
-
-// One row of the fused two-pass forward + backward, by the whole CTA.
-template <int T, int U1, int U2>
-__device__ __forceinline__ void l2_row(const RowArgs& a, const int64_t row, float2* wpart, float* bc) {
-    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    const int V = a.V;
-    const int64_t V8 = ((int64_t)V + 7) >> 3;
-    const int tailn = V & 7;
-    const float wk = a.w[row];
-    const int id = a.ids[row];
-    const bool bad = (wk != 0.f) && (id < 0 || id >= V);
-    uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
-    if (wk == 0.f || bad) {
-        if (warp == 1) prefetch_next_row(a, row, l2_policy_evict_last(), lane);
-        for (int64_t vi = t; vi < V8; vi += T) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
-        if (t == 0) {
-            write_masked_outputs(a, row);
-            if (bad) flag_status(a.status, LEAP_DEV_BAD_ID);
-        }
-        return;
-    }
-    const uint16_t* zr = a.logits + row * a.ld;
-    const uint4* zrow = reinterpret_cast<const uint4*>(zr);
-    float zy = 0.f, old = 0.f, A = 0.f;
-    if (t == 0) {
-        zy = bf16_at(zr + id);
-        old = a.old_logp[row];
-        A = a.adv[row];
-    }
-    const uint64_t keep = l2_policy_evict_last();
-    // Put the whole row's HBM reads in flight at once: pass 1 then waits on
-    // L2, not on the few loads each thread can hold in registers.
-    if (warp == 0) prefetch_row_l2(zr, V, (int64_t)1 << 40, keep, lane);
-    const float c1 = a.inv_temp * kLog2e;
-    float m = -INFINITY, s = 0.f;
-    for (int64_t v0 = t; v0 < V8; v0 += (int64_t)T * U1) {
-        uint4 x[U1];
-#pragma unroll
-        for (int u = 0; u < U1; ++u) {
-            const int64_t vi = v0 + (int64_t)u * T;
-            x[u] = (vi < V8) ? ld_stream_hint(zrow + vi, keep) : neg_inf4();
-            if (tailn && vi == V8 - 1) mask_tail(x[u], tailn);
-        }
-        const float bm = tree_max(x);
-        if (bm == -INFINITY) continue;
-        const float mn = fmaxf(m, bm);
-        const float acc = tree_exp_sum(x, c1, mn * c1);
-        s = (s == 0.f) ? acc : fmaf(s, ex2((m - mn) * c1), acc);
-        m = mn;
-    }
-    warp_lse_merge(m, s, c1);
-    if (lane == 0) wpart[warp] = make_float2(m, s);
-    __syncthreads();
-    if (warp == 0) {
-        const float2 p = (lane < T / 32) ? wpart[lane] : make_float2(-INFINITY, 0.f);
-        m = p.x;
-        s = p.y;
-        warp_lse_merge(m, s, c1);
-        if (lane == 0) {
-            const TokenLoss r = token_loss(a, m, s, zy, old, A, wk);
-            bc[0] = fmaf(m, c1, log2f(s));
-            bc[1] = a.grad_scale * r.g * a.inv_temp;
-            write_row_outputs(a, row, r, wk);
-        }
-    }
-    __syncthreads();
-    if (warp == 1) prefetch_next_row(a, row, keep, lane);
-    const float K = bc[0], coef = bc[1];
-    const uint64_t drop = l2_policy_evict_first();
-    const int64_t yv = id >> 3;
-    const int ylane = id & 7;
-    for (int64_t v0 = t; v0 < V8; v0 += (int64_t)T * U2) {
-        if (coef == 0.f) {
-#pragma unroll
-            for (int u = 0; u < U2; ++u) {
-                const int64_t vi = v0 + (int64_t)u * T;
-                if (vi < V8) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
-            }
-            continue;
-        }
-        uint4 x[U2];
-#pragma unroll
-        for (int u = 0; u < U2; ++u) {
-            const int64_t vi = v0 + (int64_t)u * T;
-            x[u] = (vi < V8) ? ld_stream_hint(zrow + vi, drop) : neg_inf4();
-        }
-#pragma unroll
-        for (int u = 0; u < U2; ++u) {
-            const int64_t vi = v0 + (int64_t)u * T;
-            if (vi < V8) store_vec(drow, vi, dlogit8(x[u], c1, K, coef, vi == yv ? ylane : -1), V8, tailn);
-        }
-    }
-}
-
-// One persistent CTA per SM walks rows blockIdx.x, + gridDim.x, ... with no
-// CTA launch between rows (the round-robin spreads masked and live rows
-// evenly; one CTA per row measured 0.845 of the copy peak against 0.871).
-template <int T, int U1, int U2>
-__global__ void __launch_bounds__(T, 1) fused_loss_l2_kernel(RowArgs a) {
-    __shared__ float2 wpart[T / 32];
-    __shared__ float bc[2];
-    for (int64_t row = blockIdx.x; row < a.N; row += gridDim.x) l2_row<T, U1, U2>(a, row, wpart, bc);
-}
-
-// ---------------------------------------------------------------------------
 // Split backward from the saved lse.  Every thread recomputes the row's scalar
 // coefficient from broadcast loads, so no block synchronisation is needed.
 // ---------------------------------------------------------------------------
@@ -698,13 +559,7 @@ cudaError_t launch_split_bwd(const RowArgs& a, cudaStream_t s) {
 cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s) {
     if (a.N == 0) return cudaSuccess;
     if (a.V <= kShortRowMaxV) return launch_short_row_loss(a, s);   // short_rows.cu
-    if (!single_read) {
-        RowArgs b = a;
-        const int64_t grid = std::min<int64_t>(a.N, (int64_t)device_sm_count());
-        b.next_stride = (int32_t)grid;   // exactly the CTA's next row
-        fused_loss_l2_kernel<kL2Threads, kL2U1, kL2U2><<<(unsigned)grid, kL2Threads, 0, s>>>(b);
-        return cudaGetLastError();
-    }
+    if (!single_read) return launch_pipe_loss(a, s);                  // loss_pipe.cu
     const int64_t V8 = ((int64_t)a.V + 7) >> 3;
     for (const FusedCfg& c : kFused) {
         const int64_t per = (V8 + c.C - 1) / c.C;

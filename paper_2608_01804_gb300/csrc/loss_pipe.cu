@@ -1,0 +1,359 @@
+// Fused forward + backward of the clipped surrogate (Eq. 3, KL skipped) with
+// the two passes over a row pipelined across consecutive rows of one SM.
+//
+// One persistent CTA per SM takes rows c, c + G, ... (G = grid size).  Its
+// warps have four roles:
+//   producer A  (one lane)  bulk-copies (TMA, 1-D) each 16 KB chunk of the
+//                           CTA's next live row into ring A, an L2 evict_last
+//                           policy on the copy so the row stays for pass 2;
+//   group A     (NA warps)  pass 1: reduces each chunk of ring A to the row's
+//                           (max, sum of exponentials), then one warp folds in
+//                           the target logit and evaluates the token's loss,
+//                           its outputs and (K, coef) for the backward, handed
+//                           to group B through a two-slot queue;
+//   producer B  (one lane)  bulk-copies the same live rows again, from L2
+//                           (evict_first), into ring B;
+//   group B     (NB warps)  pass 2: walks every row of the CTA in order,
+//                           writing zeros for masked rows and dlogits from
+//                           ring B for live ones.
+// So on every SM pass 1 of row j (HBM reads) runs beside pass 2 of row j - 1
+// (L2 re-reads and HBM writes) with the rings keeping up to (SA + SB) 16 KB
+// copies in flight, independent of the threads' registers.  HBM sees 2V
+// bytes read and 2V written per live row.
+//
+// Every wait is on an mbarrier and bounded (2 s, LEAP_DEV_TIMEOUT): after a
+// give-up the CTA's abort flag stops every role, and each producer waits
+// (bounded again) for its copies still in flight before the CTA exits.
+#include "../../include/leap.h"
+#include "leap_common.cuh"
+#include "leap_internal.h"
+#include "loss_math.cuh"
+#include "row_math.cuh"
+
+#include <algorithm>
+#include <math.h>
+#include <mutex>
+
+namespace leap {
+namespace {
+
+// 1-D bulk copy global -> own shared memory with an L2 cache policy,
+// completing on `bar` (addresses and size multiples of 16).
+__device__ __forceinline__ void bulk_g2s_hint(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_t* bar,
+                                              uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], "
+        "%4;" ::"r"(smem_addr(smem_dst)),
+        "l"(gsrc), "r"(bytes), "r"(smem_addr(bar)), "l"(policy)
+        : "memory");
+}
+
+template <int NA, int SA, int SB, int CV>
+struct PipeSmem {
+    uint4 ringA[SA][CV];
+    uint4 ringB[SB][CV];
+    uint64_t fullA[SA], emptyA[SA], fullB[SB], emptyB[SB];
+    uint64_t kcfull[2], kcempty[2];
+    float2 kc[2];            // (K = log2 of the row's normaliser in c1 units, coef) per queue slot
+    float2 wpart[2][NA];     // per-warp (max, sum) of group A, by row parity
+    int abort_flag;
+};
+
+// Barrier over `n` threads on hardware barrier `id` that also ORs a predicate
+// over them: every participant gets the same answer.
+__device__ __forceinline__ bool bar_red_or(uint32_t id, uint32_t n, bool p) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred pi, po;\n\t"
+        "setp.ne.u32 pi, %1, 0;\n\t"
+        "bar.red.or.pred po, %2, %3, pi;\n\t"
+        "selp.u32 %0, 1, 0, po;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)p), "r"(id), "r"(n)
+        : "memory");
+    return r != 0;
+}
+
+__device__ __forceinline__ bool row_live(const RowArgs& a, int64_t row) {
+    const float wk = a.w[row];
+    const int id = a.ids[row];
+    return wk != 0.f && id >= 0 && id < a.V;
+}
+
+// One producer: copies every chunk of the CTA's live rows, in order, into a
+// ring of S stages; then waits for whatever of its copies is still in flight.
+template <int S, int CV>
+__device__ __forceinline__ void pipe_produce(const RowArgs& a, uint4 (*ring)[CV], uint64_t* full,
+                                             uint64_t* empty, uint64_t policy, volatile int* abort_flag) {
+    constexpr int64_t kPipeChunk = CV * 16;
+    const int64_t G = gridDim.x;
+    const int64_t rowbytes = (int64_t)(a.V & ~7) * 2;
+    const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
+    uint32_t cnt = 0;
+    bool go = true;
+    for (int64_t row = blockIdx.x; go && row < a.N; row += G) {
+        if (!row_live(a, row)) continue;
+        const char* src = reinterpret_cast<const char*>(a.logits + row * a.ld);
+        for (int64_t k = 0; k < nch; ++k) {
+            const uint32_t s = cnt % S, ph = (cnt / S) & 1u;
+            if (!mbar_wait(&empty[s], ph ^ 1u, a.status, abort_flag)) {
+                go = false;
+                break;
+            }
+            fence_proxy_async_smem();
+            const uint32_t bytes = (uint32_t)min((int64_t)kPipeChunk, rowbytes - k * kPipeChunk);
+            mbar_arrive_expect_tx(&full[s], bytes);
+            bulk_g2s_hint(&ring[s][0], src + k * kPipeChunk, bytes, &full[s], policy);
+            ++cnt;
+        }
+    }
+    // Copies the consumers have not waited for may still be landing: wait
+    // for the last copy of every stage (returns at once for consumed ones).
+    for (uint32_t s = 0; s < (uint32_t)S && s < cnt; ++s) {
+        const uint32_t last = cnt - 1 - ((cnt - 1 - s) % S);   // last copy into stage s
+        mbar_wait_bounded<false>(&full[s], (last / S) & 1u, a.status, abort_flag);
+    }
+    if (*abort_flag) {
+        // After a give-up the waits above return at once: spin (bounded) on
+        // the stages directly so no copy outlives the CTA.
+        for (uint32_t s = 0; s < (uint32_t)S && s < cnt; ++s) {
+            const uint32_t last = cnt - 1 - ((cnt - 1 - s) % S);
+            const uint64_t t0 = globaltimer_ns();
+            while (!mbar_try_wait(&full[s], (last / S) & 1u) && globaltimer_ns() - t0 < kWaitLimitNs) {
+            }
+        }
+    }
+}
+
+template <int NA, int NB, int SA, int SB, int CV>
+__global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(RowArgs a) {
+    extern __shared__ __align__(128) unsigned char pipe_smem_raw[];
+    PipeSmem<NA, SA, SB, CV>& sm = *reinterpret_cast<PipeSmem<NA, SA, SB, CV>*>(pipe_smem_raw);
+    constexpr int64_t kPipeChunk = CV * 16;
+    constexpr int kPipeChunkVec = CV;
+    constexpr int TA = 32 * NA, TB = 32 * NB;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    volatile int* abort_flag = &sm.abort_flag;
+
+    if (threadIdx.x == 0) {
+        sm.abort_flag = 0;
+        for (int s = 0; s < SA; ++s) {
+            mbar_init(&sm.fullA[s], 1);
+            mbar_init(&sm.emptyA[s], NA);
+        }
+        for (int s = 0; s < SB; ++s) {
+            mbar_init(&sm.fullB[s], 1);
+            mbar_init(&sm.emptyB[s], NB);
+        }
+        for (int q = 0; q < 2; ++q) {
+            mbar_init(&sm.kcfull[q], 1);
+            mbar_init(&sm.kcempty[q], NB);
+        }
+        fence_mbar_init();
+    }
+    __syncthreads();
+
+    const int V = a.V;
+    const int64_t V8 = ((int64_t)V + 7) >> 3;
+    const int tailn = V & 7;
+    const int64_t V8f = (int64_t)(V >> 3);             // whole vectors, all bulk-copied
+    const int64_t rowbytes = V8f * 16;
+    const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
+    const int64_t G = gridDim.x;
+    const float c1 = a.inv_temp * kLog2e;
+
+    if (warp == 0) {
+        if (lane == 0) pipe_produce<SA, CV>(a, sm.ringA, sm.fullA, sm.emptyA, l2_policy_evict_last(), abort_flag);
+        return;
+    }
+    if (warp == 1) {
+        if (lane == 0) pipe_produce<SB, CV>(a, sm.ringB, sm.fullB, sm.emptyB, l2_policy_evict_first(), abort_flag);
+        return;
+    }
+
+    if (warp < 2 + NA) {
+        // ---- group A: pass 1 -------------------------------------------------
+        const int ta = threadIdx.x - 64, wa = warp - 2;
+        uint32_t cnt = 0, li = 0;
+        for (int64_t row = blockIdx.x; row < a.N; row += G) {
+            if (!row_live(a, row)) continue;
+            const uint16_t* zr = a.logits + row * a.ld;
+            float m = -INFINITY, s = 0.f;
+            bool ok = true;
+            for (int64_t k = 0; k < nch && ok; ++k) {
+                const uint32_t st = cnt % SA, ph = (cnt / SA) & 1u;
+                ok = mbar_wait(&sm.fullA[st], ph, a.status, abort_flag);
+                if (ok) {
+                    const int nvec = (int)(min((int64_t)kPipeChunk, rowbytes - k * kPipeChunk) >> 4);
+                    constexpr int U = (kPipeChunkVec + TA - 1) / TA;
+                    uint4 x[U];
+#pragma unroll
+                    for (int u = 0; u < U; ++u) {
+                        const int v = ta + u * TA;
+                        x[u] = v < nvec ? sm.ringA[st][v] : neg_inf4();
+                    }
+                    __syncwarp();                   // the stage is in registers: hand it back
+                    if (lane == 0) mbar_arrive(&sm.emptyA[st]);
+                    const float bm = tree_max(x);
+                    if (bm != -INFINITY) {
+                        const float mn = fmaxf(m, bm);
+                        const float acc = tree_exp_sum(x, c1, mn * c1);
+                        s = (s == 0.f) ? acc : fmaf(s, ex2((m - mn) * c1), acc);
+                        m = mn;
+                    }
+                } else {
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sm.emptyA[st]);
+                }
+                ++cnt;
+            }
+            if (ok && tailn && ta == 0) {   // the last, partial vector: not bulk-copied
+                uint4 x[1] = {ld_stream(reinterpret_cast<const uint4*>(zr) + V8f)};
+                mask_tail(x[0], tailn);
+                const float bm = tree_max(x);
+                const float mn = fmaxf(m, bm);
+                const float acc = tree_exp_sum(x, c1, mn * c1);
+                s = (s == 0.f) ? acc : fmaf(s, ex2((m - mn) * c1), acc);
+                m = mn;
+            }
+            warp_lse_merge(m, s, c1);
+            float2* wp = sm.wpart[li & 1];
+            if (lane == 0) wp[wa] = make_float2(m, s);
+            // Every warp of group A reaches this barrier once per live row,
+            // whether its chunk waits gave up or not, and all leave it with
+            // the same verdict.
+            if (bar_red_or(1, TA, !ok)) break;
+            if (wa == 0) {
+                const float2 p = (lane < NA) ? wp[lane] : make_float2(-INFINITY, 0.f);
+                m = p.x;
+                s = p.y;
+                warp_lse_merge(m, s, c1);
+                if (lane == 0) {
+                    const int id = a.ids[row];
+                    const float wk = a.w[row];
+                    const TokenLoss r = token_loss(a, m, s, bf16_at(zr + id), a.old_logp[row], a.adv[row], wk);
+                    write_row_outputs(a, row, r, wk);
+                    const uint32_t q = li & 1u;
+                    if (mbar_wait(&sm.kcempty[q], ((li >> 1) & 1u) ^ 1u, a.status, abort_flag)) {
+                        sm.kc[q] = make_float2(fmaf(m, c1, log2f(s)), a.grad_scale * r.g * a.inv_temp);
+                        mbar_arrive(&sm.kcfull[q]);
+                    }
+                }
+                __syncwarp();
+            }
+            ++li;
+        }
+        return;
+    }
+
+    // ---- group B: pass 2 over every row of the CTA, in order ------------------
+    const int tb = threadIdx.x - 32 * (2 + NA);
+    uint32_t cnt = 0, li = 0;
+    for (int64_t row = blockIdx.x; row < a.N; row += G) {
+        uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
+        const float wk = a.w[row];
+        const int id = a.ids[row];
+        if (!(wk != 0.f && id >= 0 && id < V)) {
+            for (int64_t vi = tb; vi < V8; vi += TB) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
+            if (tb == 0) {
+                write_masked_outputs(a, row);
+                if (wk != 0.f) flag_status(a.status, LEAP_DEV_BAD_ID);
+            }
+            continue;
+        }
+        const uint32_t q = li & 1u;
+        if (!mbar_wait(&sm.kcfull[q], (li >> 1) & 1u, a.status, abort_flag)) break;
+        const float2 kc = sm.kc[q];
+        const float K = kc.x, coef = kc.y;
+        const int64_t yv = id >> 3;
+        const int ylane = id & 7;
+        bool ok = true;
+        for (int64_t k = 0; k < nch && ok; ++k) {
+            const uint32_t st = cnt % SB, ph = (cnt / SB) & 1u;
+            ok = mbar_wait(&sm.fullB[st], ph, a.status, abort_flag);
+            if (ok) {
+                const int nvec = (int)(min((int64_t)kPipeChunk, rowbytes - k * kPipeChunk) >> 4);
+                constexpr int U = (kPipeChunkVec + TB - 1) / TB;
+                const int64_t g0 = k * kPipeChunkVec;
+                uint4 x[U];
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    const int v = tb + u * TB;
+                    x[u] = v < nvec ? sm.ringB[st][v] : make_uint4(0, 0, 0, 0);
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sm.emptyB[st]);
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    const int v = tb + u * TB;
+                    if (v < nvec) {
+                        const int64_t gv = g0 + v;
+                        const uint4 d = (coef == 0.f) ? make_uint4(0, 0, 0, 0)
+                                                      : dlogit8(x[u], c1, K, coef, gv == yv ? ylane : -1);
+                        st_stream(drow + gv, d);
+                    }
+                }
+            } else {
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sm.emptyB[st]);
+            }
+            ++cnt;
+        }
+        if (ok && tailn && tb == 0) {
+            uint4 x = ld_stream(reinterpret_cast<const uint4*>(a.logits + row * a.ld) + V8f);
+            const uint4 d = (coef == 0.f) ? make_uint4(0, 0, 0, 0)
+                                          : dlogit8(x, c1, K, coef, yv == V8f ? ylane : -1);
+            store_vec(drow, V8f, d, V8, tailn);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.kcempty[q]);
+        if (!ok) break;
+        ++li;
+    }
+}
+
+template <int NA, int NB, int SA, int SB, int CV>
+cudaError_t launch_pipe_cfg(const RowArgs& a, cudaStream_t s) {
+    auto kern = fused_loss_pipe_kernel<NA, NB, SA, SB, CV>;
+    const size_t dyn = sizeof(PipeSmem<NA, SA, SB, CV>);
+    static std::mutex mu;
+    static int done_dev = -1;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    {
+        std::lock_guard<std::mutex> lk(mu);
+        if (done_dev != dev) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+            if (e != cudaSuccess) return e;
+            done_dev = dev;
+        }
+    }
+    const int64_t grid = std::min<int64_t>(a.N, (int64_t)device_sm_count());
+    kern<<<(unsigned)grid, 32 * (2 + NA + NB), dyn, s>>>(a);
+    return cudaGetLastError();
+}
+
+// Measured on the single-turn workload (32,768 rows, V = 151,936; fraction of
+// the copy peak, the two-pass kernel without the pipeline 0.882 beside it):
+//   ring B depth (A 4 stages): 8 -> 0.835, 9 -> 0.853; (A 3 stages) 10 -> 0.906,
+//   11 -> 0.910: pass 2's re-reads want the deep ring;
+//   ring A depth (B 10-11): 2 -> 0.824, 3 -> 0.906-0.910, 4 -> 0.867: three
+//   16 KB copies in flight per SM keep pass 1 at its share of HBM, more only
+//   crowd pass 2's copies;
+//   chunks of 8 / 12 / 20 KB at the same ring bytes: 0.81-0.87 / 0.87-0.90 / 0.874;
+//   group A of 4 / 8 warps: 0.914 / 0.910; group B of 4 / 8 / 12 / 16 warps
+//   (A 4-8): 0.734 / 0.910-0.914 / 0.911 / 0.900;
+//   L2 policy of the pass-1 copies evict_last / normal: 0.910 / 0.909; of
+//   the pass-2 copies evict_first / normal: 0.910 / 0.891.
+constexpr int kPipeWarpsA = 4, kPipeWarpsB = 8, kPipeStagesA = 3, kPipeStagesB = 11;
+constexpr int kPipeChunkVectors = 1024;   // 16 KB per staged chunk
+
+}  // namespace
+
+cudaError_t launch_pipe_loss(const RowArgs& a, cudaStream_t s) {
+    if (a.N == 0) return cudaSuccess;
+    return launch_pipe_cfg<kPipeWarpsA, kPipeWarpsB, kPipeStagesA, kPipeStagesB, kPipeChunkVectors>(a, s);
+}
+
+}  // namespace leap

@@ -48,7 +48,7 @@ def _check_rows(out, orc, rows, V, dl=None):
                                   (30001, 30008), (60000, 60000), (100000, 100000), (151936, 151936), (151936, 152000),
                                   (200000, 200000)])
 def test_fused_loss_all_rows(V, ld, single_read):
-    """Both fused kernels (the L2 two-pass one, and with single_read every
+    """Both fused kernels (the row-pipelined one, and with single_read every
     cluster configuration, sizes 1, 2, 4, 8), ragged V and padded ld."""
     L = leap()
     L.leap_get_device_status()
@@ -190,14 +190,15 @@ def test_empty_batch():
 
 @pytest.mark.parametrize("N,pattern", [(1, "live"), (151, "random"), (152, "masked"), (153, "runs"),
                                        (1000, "live"), (3001, "runs"), (3001, "random"), (5000, "head")])
-def test_two_pass_kernel_row_partition(N, pattern):
-    """The two-pass kernel's persistent CTAs share the rows out among
-    themselves: every row is written, whatever the pattern of live and masked
-    rows and whether N is below, at or above the CTA count, and the loss
-    equals the oracle's sum over all rows."""
+def test_default_fused_kernel_row_partition(N, pattern):
+    """The default fused kernel's persistent CTAs share the rows out among
+    themselves and pipeline them (pass 1 of a live row beside pass 2 of the
+    previous one, masked rows in between): every row is written, whatever the
+    pattern of live and masked rows and whether N is below, at or above the
+    CTA count, and the loss equals the oracle's sum over all rows."""
     L = leap()
     L.leap_get_device_status()
-    V = 9000                                   # above the short-row limit: the two-pass kernel
+    V = 9000                                   # above the short-row limit: the pipelined kernel
     z, ids, old, adv, w = _inputs(N, V, seed=N % 53 + 60, sigma=3.0, spikes=0.01, old_sigma=0.3, mask_frac=0.0)
     r = np.arange(N)
     keep = {"live": np.ones(N, bool), "masked": np.zeros(N, bool), "random": np.random.default_rng(N).random(N) < 0.6,

@@ -1,7 +1,7 @@
 """GPU parity of the clipped surrogate (Eq. 3) away from its defaults: a
 sampling temperature (inv_temp = 0.7) and an asymmetric clip range
 (eps_low = 0.2, eps_high = 0.28), on every kernel that evaluates the loss or
-its gradient: the persistent two-pass fused kernel with more rows than CTAs,
+its gradient: the persistent row-pipelined fused kernel with more rows than CTAs,
 the single-read kernel at short and long rows, the forward-only loss with the
 split backward, and the fused lm-head with dhidden and dW.  Old log-probs are
 drawn around the tempered policy's own log-probs with sigma 0.3, and four
@@ -74,8 +74,10 @@ def _check(out, orc, V, dl=None):
         check_dlogits_rows(bf16_rows_to_f64(dl[:, :V]), orc, list(range(dl.shape[0])), EPS_LOW, EPS_HIGH)
 
 
-def test_two_pass_kernel_many_rows_per_cta():
-    """V = 151,936 with 400 rows: each of the 152 persistent CTAs walks two or three rows."""
+def test_default_fused_kernel_many_rows_per_cta():
+    """V = 151,936 with 400 rows: each of the 152 persistent CTAs walks two or
+    three rows, so the pass-1 / pass-2 pipeline of the default fused kernel
+    hands rows over at both parameter sets' clip edges."""
     L = leap()
     L.leap_get_device_status()
     V, N = 151936, 400
