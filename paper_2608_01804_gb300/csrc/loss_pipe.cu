@@ -4,22 +4,26 @@
 // One persistent CTA per SM takes rows c, c + G, ... (G = grid size).  Its
 // warps have four roles:
 //   producer A  (one lane)  bulk-copies (TMA, 1-D) each 16 KB chunk of the
-//                           CTA's next live row into ring A, an L2 evict_last
-//                           policy on the copy so the row stays for pass 2;
-//   group A     (NA warps)  pass 1: reduces each chunk of ring A to the row's
+//                           CTA's next live row into ring A (3 stages), an L2
+//                           evict_last policy on the copy so the row stays
+//                           for pass 2;
+//   group A     (4 warps)   pass 1: reduces each chunk of ring A to the row's
 //                           (max, sum of exponentials), then one warp folds in
 //                           the target logit and evaluates the token's loss,
 //                           its outputs and (K, coef) for the backward, handed
 //                           to group B through a two-slot queue;
 //   producer B  (one lane)  bulk-copies the same live rows again, from L2
-//                           (evict_first), into ring B;
-//   group B     (NB warps)  pass 2: walks every row of the CTA in order,
+//                           (evict_first), into ring B (11 stages);
+//   group B     (8 warps)   pass 2: walks every row of the CTA in order,
 //                           writing zeros for masked rows and dlogits from
 //                           ring B for live ones.
 // So on every SM pass 1 of row j (HBM reads) runs beside pass 2 of row j - 1
-// (L2 re-reads and HBM writes) with the rings keeping up to (SA + SB) 16 KB
-// copies in flight, independent of the threads' registers.  HBM sees 2V
-// bytes read and 2V written per live row.
+// (L2 re-reads and HBM writes), with up to 14 16 KB copies in flight
+// independent of the threads' registers, and each role loads the next row's
+// weight and id a row ahead (group A also the row's loss inputs when it
+// starts it), so no chain of dependent global loads sits between two rows.
+// HBM sees 2V bytes read and 2V written per live row, 2V written per masked
+// row.
 //
 // Every wait is on an mbarrier and bounded (2 s, LEAP_DEV_TIMEOUT): after a
 // give-up the CTA's abort flag stops every role, and each producer waits
@@ -48,10 +52,10 @@ __device__ __forceinline__ void bulk_g2s_hint(void* smem_dst, const void* gsrc, 
         : "memory");
 }
 
-template <int NA, int SA, int SB, int CV>
+template <int NA, int SA, int SB, int CVA, int CVB>
 struct PipeSmem {
-    uint4 ringA[SA][CV];
-    uint4 ringB[SB][CV];
+    uint4 ringA[SA][CVA];
+    uint4 ringB[SB][CVB];
     uint64_t fullA[SA], emptyA[SA], fullB[SB], emptyB[SB];
     uint64_t kcfull[2], kcempty[2];
     float2 kc[2];            // (K = log2 of the row's normaliser in c1 units, coef) per queue slot
@@ -74,12 +78,6 @@ __device__ __forceinline__ bool bar_red_or(uint32_t id, uint32_t n, bool p) {
     return r != 0;
 }
 
-__device__ __forceinline__ bool row_live(const RowArgs& a, int64_t row) {
-    const float wk = a.w[row];
-    const int id = a.ids[row];
-    return wk != 0.f && id >= 0 && id < a.V;
-}
-
 // One producer: copies every chunk of the CTA's live rows, in order, into a
 // ring of S stages; then waits for whatever of its copies is still in flight.
 template <int S, int CV>
@@ -91,8 +89,16 @@ __device__ __forceinline__ void pipe_produce(const RowArgs& a, uint4 (*ring)[CV]
     const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
     uint32_t cnt = 0;
     bool go = true;
+    float w_next = a.w[blockIdx.x];     // the next row's weight and id, a row ahead
+    int id_next = a.ids[blockIdx.x];
     for (int64_t row = blockIdx.x; go && row < a.N; row += G) {
-        if (!row_live(a, row)) continue;
+        const float wk = w_next;
+        const int id = id_next;
+        if (row + G < a.N) {
+            w_next = a.w[row + G];
+            id_next = a.ids[row + G];
+        }
+        if (!(wk != 0.f && id >= 0 && id < a.V)) continue;
         const char* src = reinterpret_cast<const char*>(a.logits + row * a.ld);
         for (int64_t k = 0; k < nch; ++k) {
             const uint32_t s = cnt % S, ph = (cnt / S) & 1u;
@@ -125,12 +131,10 @@ __device__ __forceinline__ void pipe_produce(const RowArgs& a, uint4 (*ring)[CV]
     }
 }
 
-template <int NA, int NB, int SA, int SB, int CV>
+template <int NA, int NB, int SA, int SB, int CVA, int CVB>
 __global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(RowArgs a) {
     extern __shared__ __align__(128) unsigned char pipe_smem_raw[];
-    PipeSmem<NA, SA, SB, CV>& sm = *reinterpret_cast<PipeSmem<NA, SA, SB, CV>*>(pipe_smem_raw);
-    constexpr int64_t kPipeChunk = CV * 16;
-    constexpr int kPipeChunkVec = CV;
+    PipeSmem<NA, SA, SB, CVA, CVB>& sm = *reinterpret_cast<PipeSmem<NA, SA, SB, CVA, CVB>*>(pipe_smem_raw);
     constexpr int TA = 32 * NA, TB = 32 * NB;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int* abort_flag = &sm.abort_flag;
@@ -158,26 +162,45 @@ __global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(
     const int tailn = V & 7;
     const int64_t V8f = (int64_t)(V >> 3);             // whole vectors, all bulk-copied
     const int64_t rowbytes = V8f * 16;
-    const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
     const int64_t G = gridDim.x;
     const float c1 = a.inv_temp * kLog2e;
 
     if (warp == 0) {
-        if (lane == 0) pipe_produce<SA, CV>(a, sm.ringA, sm.fullA, sm.emptyA, l2_policy_evict_last(), abort_flag);
+        if (lane == 0) pipe_produce<SA, CVA>(a, sm.ringA, sm.fullA, sm.emptyA, l2_policy_evict_last(), abort_flag);
         return;
     }
     if (warp == 1) {
-        if (lane == 0) pipe_produce<SB, CV>(a, sm.ringB, sm.fullB, sm.emptyB, l2_policy_evict_first(), abort_flag);
+        if (lane == 0) pipe_produce<SB, CVB>(a, sm.ringB, sm.fullB, sm.emptyB, l2_policy_evict_first(), abort_flag);
         return;
     }
 
     if (warp < 2 + NA) {
         // ---- group A: pass 1 -------------------------------------------------
         const int ta = threadIdx.x - 64, wa = warp - 2;
+        constexpr int64_t kPipeChunk = CVA * 16;
+        constexpr int kPipeChunkVec = CVA;
+        const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
         uint32_t cnt = 0, li = 0;
+        // The next row's weight and id are loaded a row ahead, and the row's
+        // own loss inputs (old log-prob, advantage, target logit) when it
+        // starts (measured: 0.914 -> 0.928 of the copy peak).
+        float w_next = a.w[blockIdx.x];
+        int id_next = a.ids[blockIdx.x];
         for (int64_t row = blockIdx.x; row < a.N; row += G) {
-            if (!row_live(a, row)) continue;
+            const float wk = w_next;
+            const int id = id_next;
+            if (row + G < a.N) {
+                w_next = a.w[row + G];
+                id_next = a.ids[row + G];
+            }
+            if (!(wk != 0.f && id >= 0 && id < V)) continue;
             const uint16_t* zr = a.logits + row * a.ld;
+            float zy = 0.f, old = 0.f, Adv = 0.f;
+            if (wa == 0 && lane == 0) {
+                zy = bf16_at(zr + id);
+                old = a.old_logp[row];
+                Adv = a.adv[row];
+            }
             float m = -INFINITY, s = 0.f;
             bool ok = true;
             for (int64_t k = 0; k < nch && ok; ++k) {
@@ -229,9 +252,7 @@ __global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(
                 s = p.y;
                 warp_lse_merge(m, s, c1);
                 if (lane == 0) {
-                    const int id = a.ids[row];
-                    const float wk = a.w[row];
-                    const TokenLoss r = token_loss(a, m, s, bf16_at(zr + id), a.old_logp[row], a.adv[row], wk);
+                    const TokenLoss r = token_loss(a, m, s, zy, old, Adv, wk);
                     write_row_outputs(a, row, r, wk);
                     const uint32_t q = li & 1u;
                     if (mbar_wait(&sm.kcempty[q], ((li >> 1) & 1u) ^ 1u, a.status, abort_flag)) {
@@ -248,11 +269,20 @@ __global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(
 
     // ---- group B: pass 2 over every row of the CTA, in order ------------------
     const int tb = threadIdx.x - 32 * (2 + NA);
+    constexpr int64_t kPipeChunk = CVB * 16;
+    constexpr int kPipeChunkVec = CVB;
+    const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
     uint32_t cnt = 0, li = 0;
+    float w_next = a.w[blockIdx.x];
+    int id_next = a.ids[blockIdx.x];
     for (int64_t row = blockIdx.x; row < a.N; row += G) {
         uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
-        const float wk = a.w[row];
-        const int id = a.ids[row];
+        const float wk = w_next;
+        const int id = id_next;
+        if (row + G < a.N) {
+            w_next = a.w[row + G];
+            id_next = a.ids[row + G];
+        }
         if (!(wk != 0.f && id >= 0 && id < V)) {
             for (int64_t vi = tb; vi < V8; vi += TB) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
             if (tb == 0) {
@@ -312,10 +342,10 @@ __global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(
     }
 }
 
-template <int NA, int NB, int SA, int SB, int CV>
+template <int NA, int NB, int SA, int SB, int CVA, int CVB>
 cudaError_t launch_pipe_cfg(const RowArgs& a, cudaStream_t s) {
-    auto kern = fused_loss_pipe_kernel<NA, NB, SA, SB, CV>;
-    const size_t dyn = sizeof(PipeSmem<NA, SA, SB, CV>);
+    auto kern = fused_loss_pipe_kernel<NA, NB, SA, SB, CVA, CVB>;
+    const size_t dyn = sizeof(PipeSmem<NA, SA, SB, CVA, CVB>);
     static std::mutex mu;
     static int done_dev = -1;
     int dev = 0;
@@ -335,7 +365,8 @@ cudaError_t launch_pipe_cfg(const RowArgs& a, cudaStream_t s) {
 }
 
 // Measured on the single-turn workload (32,768 rows, V = 151,936; fraction of
-// the copy peak, the two-pass kernel without the pipeline 0.882 beside it):
+// the copy peak; the two-pass kernel without the pipeline 0.882 beside it).
+// Before the per-row scalars were loaded a row ahead:
 //   ring B depth (A 4 stages): 8 -> 0.835, 9 -> 0.853; (A 3 stages) 10 -> 0.906,
 //   11 -> 0.910: pass 2's re-reads want the deep ring;
 //   ring A depth (B 10-11): 2 -> 0.824, 3 -> 0.906-0.910, 4 -> 0.867: three
@@ -345,7 +376,13 @@ cudaError_t launch_pipe_cfg(const RowArgs& a, cudaStream_t s) {
 //   group A of 4 / 8 warps: 0.914 / 0.910; group B of 4 / 8 / 12 / 16 warps
 //   (A 4-8): 0.734 / 0.910-0.914 / 0.911 / 0.900;
 //   L2 policy of the pass-1 copies evict_last / normal: 0.910 / 0.909; of
-//   the pass-2 copies evict_first / normal: 0.910 / 0.891.
+//   the pass-2 copies evict_first / normal: 0.910 / 0.891;
+//   pass 2 loading its row from L2 into registers (16-24 warps, 4-8 vectors
+//   in flight each) instead of through ring B: 0.69-0.77.
+// With them (this configuration 0.928-0.930):
+//   A / B stages 4 / 10, 2 / 12, 5 / 9: 0.891, 0.836, 0.825; A of 8 warps
+//   0.922, B of 12 warps 0.923; ring A of 8 KB x 5-6 or 32 KB x 2 chunks:
+//   0.867-0.896; ring B of 24 KB x 7 chunks: 0.927.
 constexpr int kPipeWarpsA = 4, kPipeWarpsB = 8, kPipeStagesA = 3, kPipeStagesB = 11;
 constexpr int kPipeChunkVectors = 1024;   // 16 KB per staged chunk
 
@@ -353,7 +390,8 @@ constexpr int kPipeChunkVectors = 1024;   // 16 KB per staged chunk
 
 cudaError_t launch_pipe_loss(const RowArgs& a, cudaStream_t s) {
     if (a.N == 0) return cudaSuccess;
-    return launch_pipe_cfg<kPipeWarpsA, kPipeWarpsB, kPipeStagesA, kPipeStagesB, kPipeChunkVectors>(a, s);
+    return launch_pipe_cfg<kPipeWarpsA, kPipeWarpsB, kPipeStagesA, kPipeStagesB, kPipeChunkVectors,
+                           kPipeChunkVectors>(a, s);
 }
 
 }  // namespace leap
