@@ -369,6 +369,14 @@ def cpu_oracle_rate_all_cores(batch, logits, ids, old, block=32):
         shm.unlink()
 
 
+def workload_config(prompts, rows, valid, world):
+    """The `config` object of both arms' JSON lines."""
+    return {"workload": WORKLOAD if prompts == 16 else "%d-prompt slice of: %s" % (prompts, WORKLOAD),
+            "rows_per_step_per_gpu": rows, "valid_tokens_per_step_per_gpu": valid,
+            "vocab": V, "logits_dtype": "bf16", "l2": "inputs larger than L2 (9.96 GB of logits "
+            "read and 9.96 GB of dlogits written per step)", "parallelism": "dp%d" % world}
+
+
 def reference_arm(args):
     """The oracle (fp64 CPU) as the reference implementation, timed per step on
     a bounded sample of the same workload; rank 0 only."""
@@ -406,7 +414,7 @@ def reference_arm(args):
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": WORKLOAD, "sample_rows_per_step": sample},
+            "config": workload_config(16, batch.N, valid_tokens(batch), args.gpus),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": "per step: rank/token oracle on the whole batch + loss fwd and dlogits on "
                                        "%d valid rows" % sample},
@@ -1032,10 +1040,7 @@ def main():
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
                 "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "f32", "data": "synthetic",
-                "config": {"workload": WORKLOAD if args.prompts == 16 else "%d-prompt slice of: %s" % (args.prompts, WORKLOAD),
-                           "rows_per_step_per_gpu": N, "valid_tokens_per_step_per_gpu": n_valid,
-                           "vocab": V, "logits_dtype": "bf16", "l2": "inputs larger than L2 (9.96 GB of logits "
-                           "read and 9.96 GB of dlogits written per step)", "parallelism": "dp%d" % world},
+                "config": workload_config(args.prompts, N, n_valid, world),
                 "roofline": roofline, "rows": rows, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": K * step.launches_per_run(pg), "clocks": clk}
         print(json.dumps(line), flush=True)
