@@ -19,9 +19,11 @@ namespace {
 
 constexpr int kMaxM = 8;
 
+// Sum over aligned segments of W lanes (W = 32: the warp; W = 16: each half).
+template <int W = 32>
 __device__ __forceinline__ float warp_sum_f(float v) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    for (int o = W / 2; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     return v;
 }
 
@@ -34,8 +36,9 @@ constexpr int kBucketBase = kCompBase + kPassBuckets * 6;
 constexpr int kNumStats = kBucketBase + kPassBuckets;
 
 // Eq. 6 and the advantage of every rollout the lane holds: the tournament
-// reward with the GRPO step, or the static-scalar baseline reward.
-template <int J>
+// reward with the GRPO step, or the static-scalar baseline reward.  A group
+// spans W aligned lanes (32, or 16 when a warp holds two groups).
+template <int J, int W = 32>
 __device__ __forceinline__ void group_reward(const RankArgs& a, int G, int M, const int (&d)[J], const int (&r)[J],
                                              const bool (&valid)[J], int dd, float (&Rv)[J], float (&Av)[J]) {
     const float gm1 = (float)(G - 1);
@@ -64,9 +67,9 @@ __device__ __forceinline__ void group_reward(const RankArgs& a, int G, int M, co
                 hi = fmaxf(hi, Rv[j]);
             }
         }
-        const float mean = warp_sum_f(sum) / (float)G;
+        const float mean = warp_sum_f<W>(sum) / (float)G;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
+        for (int o = W / 2; o > 0; o >>= 1) {
             lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
             hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
         }
@@ -74,7 +77,7 @@ __device__ __forceinline__ void group_reward(const RankArgs& a, int G, int M, co
 #pragma unroll
         for (int j = 0; j < J; ++j)
             if (valid[j]) ss += (Rv[j] - mean) * (Rv[j] - mean);
-        const float stdv = sqrtf(warp_sum_f(ss) / den);
+        const float stdv = sqrtf(warp_sum_f<W>(ss) / den);
 #pragma unroll
         for (int j = 0; j < J; ++j)
             Av[j] = (a.norm == 1) ? Rv[j] : ((hi == lo) ? 0.f : (Rv[j] - mean) / (stdv + a.eps_std));
@@ -136,6 +139,86 @@ __device__ __forceinline__ void group_stats(long long* cnt, int G, int M, bool g
 #pragma unroll
         for (int k = 0; k < 6; ++k) c[kCompBase + bucket * 6 + k] += comp[k];
         c[kBucketBase + bucket] += 1;
+    }
+    __syncwarp();
+}
+
+// group_stats for a warp holding two groups of 64 (lanes 0-15 the first,
+// 16-31 the second; J = 4 rollouts per lane): each lane counts its own
+// rollouts, and one warp reduction adds two counters for both groups at once
+// (8-bit fields: a group holds at most 64), so a counter costs half a
+// reduction instead of J ballots.  Lane 0 adds both groups' counts.
+template <int MB>
+__device__ __forceinline__ void group_stats_quad(long long* cnt, int M, bool gate, int n_fail, bool own,
+                                                 const bool (&valid)[4], const bool (&bad)[4], const int (&pt0)[4],
+                                                 const int (&T)[4], const int (&r)[4], const float (&Av)[4],
+                                                 int lane) {
+    constexpr int G = 64;
+    constexpr int NC = 10 + (MB - 1);   // nonzero, first, later, failed_on, comp[6], by_turn[1..MB-1]
+    int loc[NC];
+#pragma unroll
+    for (int c = 0; c < NC; ++c) loc[c] = 0;
+    int turns = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const bool ok = valid[j] && !bad[j];
+        const int pt = pt0[j];
+        const bool nz = valid[j] && Av[j] != 0.f;
+        loc[0] += nz;
+        loc[1] += ok && pt == 1;
+        loc[2] += ok && gate && pt >= 2;
+        loc[3] += ok && gate && pt != 1;
+        const int kind = (r[j] == M) ? 0 : ((r[j] > 0) ? 1 : 2);
+        const int cat = nz ? kind * 2 + (Av[j] < 0.f ? 1 : 0) : -1;
+#pragma unroll
+        for (int c = 0; c < 6; ++c) loc[4 + c] += (cat == c);
+#pragma unroll
+        for (int m = 1; m < MB; ++m) loc[9 + m] += ok && gate && pt == m + 1;
+        turns += valid[j] ? T[j] : 0;
+    }
+    const int half = lane >> 4;
+    int tot[2][NC];
+#pragma unroll
+    for (int c = 0; c < NC; c += 2) {
+        const unsigned v = ((unsigned)loc[c] << (8 * half)) |
+                           (c + 1 < NC ? ((unsigned)loc[c + 1] << (16 + 8 * half)) : 0u);
+        const unsigned s2 = __reduce_add_sync(0xffffffffu, v);
+        tot[0][c] = (int)(s2 & 0xffu);
+        tot[1][c] = (int)((s2 >> 8) & 0xffu);
+        if (c + 1 < NC) {
+            tot[0][c + 1] = (int)((s2 >> 16) & 0xffu);
+            tot[1][c + 1] = (int)(s2 >> 24);
+        }
+    }
+    const unsigned ts = __reduce_add_sync(0xffffffffu, (unsigned)turns << (16 * half));
+    const bool gate1 = __shfl_sync(0xffffffffu, gate, 16);
+    const int n_fail1 = __shfl_sync(0xffffffffu, n_fail, 16);
+    const bool own1 = __shfl_sync(0xffffffffu, own, 16);
+    if (lane == 0) {
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+            if (!(g ? own1 : own)) continue;
+            const bool gt = g ? gate1 : gate;
+            const int nf = g ? n_fail1 : n_fail;
+            const int* t = tot[g];
+            long long* c = cnt;
+            c[0] += 1;
+            c[1] += gt;
+            c[2] += G;
+            c[3] += t[0];
+            c[4] += t[1];
+            c[5] += t[2];
+            c[6] += (t[2] > 0);
+            c[7] += t[3];
+            c[8] += g ? (int)(ts >> 16) : (int)(ts & 0xffffu);
+            c[9] += t[1];
+#pragma unroll
+            for (int m = 1; m < MB; ++m) c[9 + m] += t[9 + m];
+            const int bucket = min(kPassBuckets - 1, (kPassBuckets * (G - nf)) / G);
+#pragma unroll
+            for (int k = 0; k < 6; ++k) c[kCompBase + bucket * 6 + k] += t[4 + k];
+            c[kBucketBase + bucket] += 1;
+        }
     }
     __syncwarp();
 }
@@ -521,13 +604,14 @@ __global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs
     if (a.stats) flush_stats(a, sst);
 }
 
-// G = 64 with the paper's comparator and the tournament reward, without
-// counters: a warp takes two groups per iteration (128 consecutive rollouts),
-// lane l holding rollouts 4l .. 4l + 3 (lanes 0-15 the first group, 16-31 the
-// second).  Each outcome array is one 4-byte load and each output array one
-// 16-byte store per lane (the turn advantages as M float4), and the two
-// groups' sums share warp reductions (the failure counts packed in 16-bit
-// halves, the tier histograms and squared net scores one reduction per group):
+// G = 64 with the paper's comparator (either reward, with or without the
+// training counters): a warp takes two groups per iteration (128 consecutive
+// rollouts), lane l holding rollouts 4l .. 4l + 3 (lanes 0-15 the first group,
+// 16-31 the second).  Each outcome array is one 4-byte load and each output
+// array one 16-byte store per lane (the turn advantages as M float4), and the
+// two groups' sums share warp reductions (the failure counts packed in 16-bit
+// halves, the tier histograms and squared net scores one reduction per group,
+// the static reward's sums over half-warps, the counters two per reduction):
 // half the memory instructions and loop overhead of the pair kernel per
 // rollout.
 constexpr int kQuadMinBlocks = 4;
@@ -539,6 +623,12 @@ __global__ void __launch_bounds__(256, kQuadMinBlocks) rank_quad_kernel(RankArgs
 
     const int64_t npairs = ((int64_t)a.num_groups + 1) / 2;
     const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    const int wib = threadIdx.x >> 5;
+    __shared__ long long sst[8][kNumStats];
+    if (a.stats) {
+        for (int k = lane; k < kNumStats; k += 32) sst[wib][k] = 0;
+        __syncwarp();
+    }
     for (int64_t pr = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); pr < npairs; pr += warps) {
         const int64_t group = 2 * pr + half;
         const bool own = group < a.num_groups;   // the last pair may hold one group
@@ -621,7 +711,7 @@ __global__ void __launch_bounds__(256, kQuadMinBlocks) rank_quad_kernel(RankArgs
         const int dd = half ? dd1 : dd0;
 
         float Rv[J], Av[J];
-        group_reward<J>(a, G, M, d, r, valid, dd, Rv, Av);
+        group_reward<J, 16>(a, G, M, d, r, valid, dd, Rv, Av);
 
         if (own) {
             if (a.n_worse) *reinterpret_cast<int4*>(a.n_worse + i0) = make_int4(nw[0], nw[1], nw[2], nw[3]);
@@ -650,7 +740,9 @@ __global__ void __launch_bounds__(256, kQuadMinBlocks) rank_quad_kernel(RankArgs
             for (int q = 0; q < M; ++q) ta[q] = make_float4(tv[4 * q], tv[4 * q + 1], tv[4 * q + 2], tv[4 * q + 3]);
             if ((lane & 15) == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
         }
+        if (a.stats) group_stats_quad<M>(sst[wib], M, gate, n_fail, own, valid, bad, pt0, T, r, Av, lane);
     }
+    if (a.stats) flush_stats(a, sst);
 }
 
 template <int MC>
@@ -1061,7 +1153,7 @@ cudaError_t launch_rank_advantages(const RankArgs& a, cudaStream_t s) {
     if (a.num_groups == 0) return cudaSuccess;
     // Groups of 64 (the quad kernel): 4-byte aligned byte arrays and 16-byte
     // aligned 4-byte arrays (every lane's four rollouts start at a multiple of 4).
-    const bool quad = a.cmp == 0 && a.reward == 0 && !a.stats && a.G == 64 && aligned_to(a.pass_turn, 4) &&
+    const bool quad = a.cmp == 0 && a.G == 64 && aligned_to(a.pass_turn, 4) &&
                       aligned_to(a.num_turns, 4) && aligned_to(a.T_eff, 4) && aligned_to(a.r_out, 4) &&
                       aligned_to(a.n_worse, 16) && aligned_to(a.n_better, 16) && aligned_to(a.R, 16) &&
                       aligned_to(a.A, 16) && aligned_to(a.turn_adv, 16);

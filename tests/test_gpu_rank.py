@@ -310,3 +310,53 @@ def test_quad_pair_and_generic_kernels_agree_at_64(M):
             assert torch.equal(quad[k], other[k]), k
     orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, tau[0], tau[1], 0.8)
     _compare(quad, orc, M)
+
+
+@pytest.mark.parametrize("reward", [0, 1])
+@pytest.mark.parametrize("M", [1, 3, 8])
+def test_quad_pair_and_generic_counters_and_rewards_at_64(M, reward):
+    """The quad kernel also serves the training counters (two groups' counts
+    in one warp reduction) and the static-scalar reward (half-warp sums): on
+    an odd group count, with one malformed outcome and a computed gate, the
+    counters of the quad, pair and generic kernels all equal the oracle's, the
+    integer outputs agree bit for bit, and the advantages match the oracle."""
+    G = 64
+    rng = np.random.default_rng(13 * M + reward)
+    groups = 37
+    n = groups * G
+    nt = rng.integers(1, M + 1, size=n).astype(np.int8)
+    pt = np.minimum(np.where(rng.random(n) < 0.5, rng.integers(1, M + 1, size=n), 0), nt).astype(np.int8)
+    pt[70] = M + 1
+    L = leap()
+    dev = torch.device("cuda")
+    pt_d, nt_d = torch.as_tensor(pt, device=dev), torch.as_tensor(nt, device=dev)
+    tau = (16, 48)
+    L.leap_get_device_status()                      # clears the sticky flags
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, tau[0], tau[1], 0.8, reward=reward,
+                            static_c=0.5)
+    exp = O.rank_stats(orc, pt.reshape(-1, G), M)
+    results = []
+    for shift4, shift1 in ((0, 0), (2, 2), (1, 1)):   # quad; pair (8 / 2-byte offsets); generic (4 / 1-byte)
+        off = lambda k, dt, sh: torch.empty(k + sh, dtype=dt, device=dev)[sh:]
+        out = dict(gate=off(groups, torch.uint8, shift1), r=off(n, torch.uint8, shift1),
+                   n_worse=off(n, torch.int32, shift4), n_better=off(n, torch.int32, shift4),
+                   R=off(n, torch.float32, shift4), A=off(n, torch.float32, shift4),
+                   turn_adv=off(n * M, torch.float32, shift4), T_eff=off(n, torch.uint8, shift1))
+        st = L.rank_stats_tensor("cuda")
+        res = L.leap_group_rank_advantages(pt_d, nt_d, G=G, M=M, tau_min=tau[0], tau_max=tau[1], gamma=0.8,
+                                           out=out, stats=st, reward=reward, static_c=0.5)
+        assert L.read_rank_stats(st) == exp
+        results.append(res)
+    torch.cuda.synchronize()
+    assert L.leap_get_device_status() == L.LEAP_DEV_BAD_OUTCOME   # read (and cleared) here
+    for other in results[1:]:
+        for k in ("gate", "r", "T_eff", "n_worse", "n_better"):
+            assert torch.equal(results[0][k], other[k]), k
+    for res in results:
+        if reward == 0:
+            _compare(res, orc, M)
+        else:
+            np.testing.assert_allclose(res["R"].cpu().numpy(), orc["R"].reshape(-1), rtol=0, atol=1e-7)
+            assert np.max(np.abs(res["A"].cpu().numpy() - orc["A"].reshape(-1))) <= TOL_ADV
+            ta = res["turn_adv"].cpu().numpy().reshape(-1, M)
+            assert np.max(np.abs(ta - orc["turn_adv"].reshape(-1, M))) <= TOL_ADV
