@@ -147,9 +147,19 @@ __device__ __forceinline__ void group_stats(long long* cnt, int G, int M, bool g
 // 16-31 the second; J = 4 rollouts per lane): each lane counts its own
 // rollouts, and one warp reduction adds two counters for both groups at once
 // (8-bit fields: a group holds at most 64), so a counter costs half a
-// reduction instead of J ballots.  Lane 0 adds both groups' counts.
+// reduction instead of J ballots.  The running totals stay in registers:
+// the scalar counters in every lane (warp-uniform), the Fig. 4 counters of
+// pass-rate bucket b in lane b; quad_stats_flush writes them to the warp's
+// shared-memory row once.  A warp sees at most 2^31 / (4 x 64) groups per
+// launch, so 32-bit totals cannot overflow.
 template <int MB>
-__device__ __forceinline__ void group_stats_quad(long long* cnt, int M, bool gate, int n_fail, bool own,
+struct QuadStats {
+    uint32_t sc[9 + MB];   // leap_rank_stats_t's scalar counters, in its order (passes at turns <= MB)
+    uint32_t bk[7];        // this lane's bucket: composition [type][sign], then groups
+};
+
+template <int MB>
+__device__ __forceinline__ void group_stats_quad(QuadStats<MB>& q, int M, bool gate, int n_fail, bool own,
                                                  const bool (&valid)[4], const bool (&bad)[4], const int (&pt0)[4],
                                                  const int (&T)[4], const int (&r)[4], const float (&Av)[4],
                                                  int lane) {
@@ -194,31 +204,43 @@ __device__ __forceinline__ void group_stats_quad(long long* cnt, int M, bool gat
     const bool gate1 = __shfl_sync(0xffffffffu, gate, 16);
     const int n_fail1 = __shfl_sync(0xffffffffu, n_fail, 16);
     const bool own1 = __shfl_sync(0xffffffffu, own, 16);
-    if (lane == 0) {
+    const bool gate0 = __shfl_sync(0xffffffffu, gate, 0);
+    const int n_fail0 = __shfl_sync(0xffffffffu, n_fail, 0);
+    const bool own0 = __shfl_sync(0xffffffffu, own, 0);
 #pragma unroll
-        for (int g = 0; g < 2; ++g) {
-            if (!(g ? own1 : own)) continue;
-            const bool gt = g ? gate1 : gate;
-            const int nf = g ? n_fail1 : n_fail;
-            const int* t = tot[g];
-            long long* c = cnt;
-            c[0] += 1;
-            c[1] += gt;
-            c[2] += G;
-            c[3] += t[0];
-            c[4] += t[1];
-            c[5] += t[2];
-            c[6] += (t[2] > 0);
-            c[7] += t[3];
-            c[8] += g ? (int)(ts >> 16) : (int)(ts & 0xffffu);
-            c[9] += t[1];
+    for (int g = 0; g < 2; ++g) {
+        if (!(g ? own1 : own0)) continue;
+        const bool gt = g ? gate1 : gate0;
+        const int nf = g ? n_fail1 : n_fail0;
+        const int* t = tot[g];
+        q.sc[0] += 1;
+        q.sc[1] += gt;
+        q.sc[2] += G;
+        q.sc[3] += t[0];
+        q.sc[4] += t[1];
+        q.sc[5] += t[2];
+        q.sc[6] += (t[2] > 0);
+        q.sc[7] += t[3];
+        q.sc[8] += g ? (ts >> 16) : (ts & 0xffffu);
+        q.sc[9] += t[1];
 #pragma unroll
-            for (int m = 1; m < MB; ++m) c[9 + m] += t[9 + m];
-            const int bucket = min(kPassBuckets - 1, (kPassBuckets * (G - nf)) / G);
+        for (int m = 1; m < MB; ++m) q.sc[9 + m] += t[9 + m];
+        if (lane == min(kPassBuckets - 1, (kPassBuckets * (G - nf)) / G)) {
 #pragma unroll
-            for (int k = 0; k < 6; ++k) c[kCompBase + bucket * 6 + k] += t[4 + k];
-            c[kBucketBase + bucket] += 1;
+            for (int k = 0; k < 6; ++k) q.bk[k] += t[4 + k];
+            q.bk[6] += 1;
         }
+    }
+}
+
+// The warp's running counters into its row of shared-memory counters.
+template <int MB>
+__device__ __forceinline__ void quad_stats_flush(const QuadStats<MB>& q, long long* cnt, int lane) {
+    if (lane == 0)
+        for (int k = 0; k < kCompBase; ++k) cnt[k] = k < 9 + MB ? (long long)q.sc[k] : 0;
+    if (lane < kPassBuckets) {
+        for (int k = 0; k < 6; ++k) cnt[kCompBase + lane * 6 + k] = q.bk[k];
+        cnt[kBucketBase + lane] = q.bk[6];
     }
     __syncwarp();
 }
@@ -614,9 +636,11 @@ __global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs
 // the static reward's sums over half-warps, the counters two per reduction):
 // half the memory instructions and loop overhead of the pair kernel per
 // rollout.
-constexpr int kQuadMinBlocks = 4;
-template <int MC>
-__global__ void __launch_bounds__(256, kQuadMinBlocks) rank_quad_kernel(RankArgs a) {
+// Blocks of 256 per SM the register budget is cut for: 4 without counters
+// (64 registers); with them (the running totals take 9 + M + 7 registers) 3.
+constexpr int kQuadMinBlocks = 4, kQuadStatsMinBlocks = 3;
+template <int MC, bool STATS>
+__global__ void __launch_bounds__(256, STATS ? kQuadStatsMinBlocks : kQuadMinBlocks) rank_quad_kernel(RankArgs a) {
     constexpr int J = 4, M = MC, G = 64;
     const int lane = threadIdx.x & 31;
     const int half = lane >> 4;
@@ -625,9 +649,12 @@ __global__ void __launch_bounds__(256, kQuadMinBlocks) rank_quad_kernel(RankArgs
     const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
     const int wib = threadIdx.x >> 5;
     __shared__ long long sst[8][kNumStats];
-    if (a.stats) {
-        for (int k = lane; k < kNumStats; k += 32) sst[wib][k] = 0;
-        __syncwarp();
+    QuadStats<MC> qs;
+    if (STATS) {
+#pragma unroll
+        for (int k = 0; k < 9 + MC; ++k) qs.sc[k] = 0;
+#pragma unroll
+        for (int k = 0; k < 7; ++k) qs.bk[k] = 0;
     }
     for (int64_t pr = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); pr < npairs; pr += warps) {
         const int64_t group = 2 * pr + half;
@@ -740,17 +767,22 @@ __global__ void __launch_bounds__(256, kQuadMinBlocks) rank_quad_kernel(RankArgs
             for (int q = 0; q < M; ++q) ta[q] = make_float4(tv[4 * q], tv[4 * q + 1], tv[4 * q + 2], tv[4 * q + 3]);
             if ((lane & 15) == 0 && a.gate_out) a.gate_out[group] = gate ? 1 : 0;
         }
-        if (a.stats) group_stats_quad<M>(sst[wib], M, gate, n_fail, own, valid, bad, pt0, T, r, Av, lane);
+        if (STATS) group_stats_quad<M>(qs, M, gate, n_fail, own, valid, bad, pt0, T, r, Av, lane);
     }
-    if (a.stats) flush_stats(a, sst);
+    if (STATS) {
+        quad_stats_flush(qs, sst[wib], lane);
+        flush_stats(a, sst);
+    }
 }
 
 template <int MC>
 cudaError_t launch_quad(const RankArgs& a, cudaStream_t s) {
     const int warps = 8;
     const int64_t pairs = ((int64_t)a.num_groups + 1) / 2;
-    const int64_t blocks = std::min<int64_t>((pairs + warps - 1) / warps, (int64_t)device_sm_count() * kQuadMinBlocks);
-    rank_quad_kernel<MC><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
+    const int per_sm = a.stats ? kQuadStatsMinBlocks : kQuadMinBlocks;
+    const int64_t blocks = std::min<int64_t>((pairs + warps - 1) / warps, (int64_t)device_sm_count() * per_sm);
+    if (a.stats) rank_quad_kernel<MC, true><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
+    else rank_quad_kernel<MC, false><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
     return cudaGetLastError();
 }
 
