@@ -7,11 +7,12 @@
 //                           CTA's next live row into ring A (3 stages), an L2
 //                           evict_last policy on the copy so the row stays
 //                           for pass 2;
-//   group A     (4 warps)   pass 1: reduces each chunk of ring A to the row's
-//                           (max, sum of exponentials), then one warp folds in
-//                           the target logit and evaluates the token's loss,
-//                           its outputs and (K, coef) for the backward, handed
-//                           to group B through a two-slot queue;
+//   group A     (4 warps)   pass 1: reduces each chunk of ring A to per-warp
+//                           (max, sum of exponentials) and goes straight on
+//                           to the next live row;
+//   finishing   (one warp)  merges group A's partials of a row, evaluates the
+//                           token's loss and outputs, and hands (K, coef) for
+//                           the backward to group B through a two-slot queue;
 //   producer B  (one lane)  bulk-copies the same live rows again, from L2
 //                           (evict_first), into ring B (11 stages);
 //   group B     (8 warps)   pass 2: walks every row of the CTA in order,
@@ -20,8 +21,11 @@
 // So on every SM pass 1 of row j (HBM reads) runs beside pass 2 of row j - 1
 // (L2 re-reads and HBM writes), with up to 14 16 KB copies in flight
 // independent of the threads' registers, and each role loads the next row's
-// weight and id a row ahead (group A also the row's loss inputs when it
-// starts it), so no chain of dependent global loads sits between two rows.
+// weight and id a row ahead (the finishing warp also the row's loss inputs
+// before it waits for the row's partials), so no chain of dependent global
+// loads and no block-wide barrier sits between two rows; group A starts a
+// row only once group B has finished the row two before it, which keeps the
+// rows between the passes in L2.
 // HBM sees 2V bytes read and 2V written per live row, 2V written per masked
 // row.
 //
@@ -60,23 +64,9 @@ struct PipeSmem {
     uint64_t kcfull[2], kcempty[2];
     float2 kc[2];            // (K = log2 of the row's normaliser in c1 units, coef) per queue slot
     float2 wpart[2][NA];     // per-warp (max, sum) of group A, by row parity
+    uint64_t wfull[2], wempty[2];   // group A -> finishing warp, by row parity
     int abort_flag;
 };
-
-// Barrier over `n` threads on hardware barrier `id` that also ORs a predicate
-// over them: every participant gets the same answer.
-__device__ __forceinline__ bool bar_red_or(uint32_t id, uint32_t n, bool p) {
-    uint32_t r;
-    asm volatile(
-        "{\n\t.reg .pred pi, po;\n\t"
-        "setp.ne.u32 pi, %1, 0;\n\t"
-        "bar.red.or.pred po, %2, %3, pi;\n\t"
-        "selp.u32 %0, 1, 0, po;\n\t}"
-        : "=r"(r)
-        : "r"((uint32_t)p), "r"(id), "r"(n)
-        : "memory");
-    return r != 0;
-}
 
 // One producer: copies every chunk of the CTA's live rows, in order, into a
 // ring of S stages; then waits for whatever of its copies is still in flight.
@@ -132,7 +122,7 @@ __device__ __forceinline__ void pipe_produce(const RowArgs& a, uint4 (*ring)[CV]
 }
 
 template <int NA, int NB, int SA, int SB, int CVA, int CVB>
-__global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(RowArgs a) {
+__global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(RowArgs a) {
     extern __shared__ __align__(128) unsigned char pipe_smem_raw[];
     PipeSmem<NA, SA, SB, CVA, CVB>& sm = *reinterpret_cast<PipeSmem<NA, SA, SB, CVA, CVB>*>(pipe_smem_raw);
     constexpr int TA = 32 * NA, TB = 32 * NB;
@@ -152,6 +142,8 @@ __global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(
         for (int q = 0; q < 2; ++q) {
             mbar_init(&sm.kcfull[q], 1);
             mbar_init(&sm.kcempty[q], NB);
+            mbar_init(&sm.wfull[q], NA);
+            mbar_init(&sm.wempty[q], 1);
         }
         fence_mbar_init();
     }
@@ -174,16 +166,57 @@ __global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(
         return;
     }
 
-    if (warp < 2 + NA) {
+    constexpr int A0 = 3;   // first warp of group A
+    if (warp == 2) {
+        // ---- finishing warp: merges group A's partials, evaluates the token's
+        // loss and hands (K, coef) to group B, while group A goes on to the
+        // next row.
+        uint32_t li = 0;
+        float w_next = a.w[blockIdx.x];
+        int id_next = a.ids[blockIdx.x];
+        for (int64_t row = blockIdx.x; row < a.N; row += G) {
+            const float wk = w_next;
+            const int id = id_next;
+            if (row + G < a.N) {
+                w_next = a.w[row + G];
+                id_next = a.ids[row + G];
+            }
+            if (!(wk != 0.f && id >= 0 && id < V)) continue;
+            float zy = 0.f, old = 0.f, Adv = 0.f;
+            if (lane == 0) {
+                zy = bf16_at(a.logits + row * a.ld + id);
+                old = a.old_logp[row];
+                Adv = a.adv[row];
+            }
+            const uint32_t q = li & 1u;
+            if (!mbar_wait(&sm.wfull[q], (li >> 1) & 1u, a.status, abort_flag)) break;
+            const float2 p = (lane < NA) ? sm.wpart[q][lane] : make_float2(-INFINITY, 0.f);
+            float m = p.x, s = p.y;
+            warp_lse_merge(m, s, c1);
+            if (lane == 0) {
+                const TokenLoss r = token_loss(a, m, s, zy, old, Adv, wk);
+                write_row_outputs(a, row, r, wk);
+                if (mbar_wait(&sm.kcempty[q], ((li >> 1) & 1u) ^ 1u, a.status, abort_flag)) {
+                    sm.kc[q] = make_float2(fmaf(m, c1, log2f(s)), a.grad_scale * r.g * a.inv_temp);
+                    mbar_arrive(&sm.kcfull[q]);
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.wempty[q]);
+            ++li;
+        }
+        return;
+    }
+    if (warp < A0 + NA) {
         // ---- group A: pass 1 -------------------------------------------------
-        const int ta = threadIdx.x - 64, wa = warp - 2;
+        const int ta = threadIdx.x - 32 * A0, wa = warp - A0;
         constexpr int64_t kPipeChunk = CVA * 16;
         constexpr int kPipeChunkVec = CVA;
         const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
         uint32_t cnt = 0, li = 0;
-        // The next row's weight and id are loaded a row ahead, and the row's
-        // own loss inputs (old log-prob, advantage, target logit) when it
-        // starts (measured: 0.914 -> 0.928 of the copy peak).
+        // The next row's weight and id are loaded a row ahead (every role does;
+        // with the finishing warp's early loads of the loss inputs, measured
+        // 0.914 -> 0.928 of the copy peak).
         float w_next = a.w[blockIdx.x];
         int id_next = a.ids[blockIdx.x];
         for (int64_t row = blockIdx.x; row < a.N; row += G) {
@@ -195,11 +228,14 @@ __global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(
             }
             if (!(wk != 0.f && id >= 0 && id < V)) continue;
             const uint16_t* zr = a.logits + row * a.ld;
-            float zy = 0.f, old = 0.f, Adv = 0.f;
-            if (wa == 0 && lane == 0) {
-                zy = bf16_at(zr + id);
-                old = a.old_logp[row];
-                Adv = a.adv[row];
+            // Start live row li once group B has finished row li - 2 (the
+            // queue slot's release): pass 1 stays at most about one row
+            // ahead of pass 2, so the rows between them still sit in L2 when
+            // pass 2 re-reads them (long masked runs would otherwise let it
+            // run three rows ahead and the re-reads miss).
+            if (li >= 2) {
+                if (lane == 0) mbar_wait(&sm.kcempty[li & 1u], ((li >> 1) & 1u) ^ 1u, a.status, abort_flag);
+                __syncwarp();
             }
             float m = -INFINITY, s = 0.f;
             bool ok = true;
@@ -240,35 +276,24 @@ __global__ void __launch_bounds__(32 * (2 + NA + NB), 1) fused_loss_pipe_kernel(
                 m = mn;
             }
             warp_lse_merge(m, s, c1);
-            float2* wp = sm.wpart[li & 1];
-            if (lane == 0) wp[wa] = make_float2(m, s);
-            // Every warp of group A reaches this barrier once per live row,
-            // whether its chunk waits gave up or not, and all leave it with
-            // the same verdict.
-            if (bar_red_or(1, TA, !ok)) break;
-            if (wa == 0) {
-                const float2 p = (lane < NA) ? wp[lane] : make_float2(-INFINITY, 0.f);
-                m = p.x;
-                s = p.y;
-                warp_lse_merge(m, s, c1);
-                if (lane == 0) {
-                    const TokenLoss r = token_loss(a, m, s, zy, old, Adv, wk);
-                    write_row_outputs(a, row, r, wk);
-                    const uint32_t q = li & 1u;
-                    if (mbar_wait(&sm.kcempty[q], ((li >> 1) & 1u) ^ 1u, a.status, abort_flag)) {
-                        sm.kc[q] = make_float2(fmaf(m, c1, log2f(s)), a.grad_scale * r.g * a.inv_temp);
-                        mbar_arrive(&sm.kcfull[q]);
-                    }
+            // Hand the warp's partial to the finishing warp (its slot of this
+            // row parity is free once that warp merged the row two rows back).
+            if (!ok) break;
+            if (lane == 0) {
+                const uint32_t q = li & 1u;
+                if (mbar_wait(&sm.wempty[q], ((li >> 1) & 1u) ^ 1u, a.status, abort_flag)) {
+                    sm.wpart[q][wa] = make_float2(m, s);
+                    mbar_arrive(&sm.wfull[q]);
                 }
-                __syncwarp();
             }
+            __syncwarp();
             ++li;
         }
         return;
     }
 
     // ---- group B: pass 2 over every row of the CTA, in order ------------------
-    const int tb = threadIdx.x - 32 * (2 + NA);
+    const int tb = threadIdx.x - 32 * (A0 + NA);
     constexpr int64_t kPipeChunk = CVB * 16;
     constexpr int kPipeChunkVec = CVB;
     const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
@@ -360,7 +385,7 @@ cudaError_t launch_pipe_cfg(const RowArgs& a, cudaStream_t s) {
         }
     }
     const int64_t grid = std::min<int64_t>(a.N, (int64_t)device_sm_count());
-    kern<<<(unsigned)grid, 32 * (2 + NA + NB), dyn, s>>>(a);
+    kern<<<(unsigned)grid, 32 * (3 + NA + NB), dyn, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -383,6 +408,11 @@ cudaError_t launch_pipe_cfg(const RowArgs& a, cudaStream_t s) {
 //   A / B stages 4 / 10, 2 / 12, 5 / 9: 0.891, 0.836, 0.825; A of 8 warps
 //   0.922, B of 12 warps 0.923; ring A of 8 KB x 5-6 or 32 KB x 2 chunks:
 //   0.867-0.896; ring B of 24 KB x 7 chunks: 0.927.
+// A finishing warp taking the row-end merge and loss off group A (which no
+// longer meets at a block barrier per row): 0.926 -> 0.931 (4 / 10 stages
+// with it 0.840, group A of 8 warps 0.918), but the multi-turn step (long
+// masked runs) 0.904 -> 0.890 as pass 1 ran further ahead of pass 2; with
+// pass 1's lead bounded to two rows of queue: 0.933 and 0.910.
 constexpr int kPipeWarpsA = 4, kPipeWarpsB = 8, kPipeStagesA = 3, kPipeStagesB = 11;
 constexpr int kPipeChunkVectors = 1024;   // 16 KB per staged chunk
 
