@@ -81,7 +81,7 @@ struct LossWorkspace {
     long long* part_clip;
     int64_t nblk;
 };
-constexpr int64_t kReduceRowsPerBlock = 4096;
+constexpr int64_t kReduceRowsPerBlock = 512;
 size_t loss_workspace_bytes(int64_t N);
 LossWorkspace carve_loss_workspace(void* base, int64_t N);
 

@@ -357,74 +357,83 @@ __global__ void __launch_bounds__(512) split_bwd_kernel(RowArgs a) {
 // ---------------------------------------------------------------------------
 constexpr int kRedThreads = 256;
 
-template <typename Tv>
-__device__ __forceinline__ Tv block_sum_fixed(Tv v, Tv* sh) {
-    sh[threadIdx.x] = v;
-    __syncthreads();
-    for (int o = blockDim.x / 2; o > 0; o >>= 1) {
-        if ((int)threadIdx.x < o) sh[threadIdx.x] += sh[threadIdx.x + o];
-        __syncthreads();
+// The four sums of the loss reduction, over a block in a fixed order: a
+// shuffle tree within each warp, then thread 0 adds the warps' sums in warp
+// order (one block barrier).  The result is valid in thread 0.
+struct LossSums {
+    double loss, rho;
+    long long live, clip;
+};
+__device__ __forceinline__ LossSums block_sums_fixed(LossSums v) {
+    __shared__ LossSums sh[kRedThreads / 32];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        v.loss += __shfl_down_sync(0xffffffffu, v.loss, o);
+        v.rho += __shfl_down_sync(0xffffffffu, v.rho, o);
+        v.live += __shfl_down_sync(0xffffffffu, v.live, o);
+        v.clip += __shfl_down_sync(0xffffffffu, v.clip, o);
     }
-    const Tv r = sh[0];
+    if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = v;
     __syncthreads();
-    return r;
+    LossSums t = {0.0, 0.0, 0, 0};
+    if (threadIdx.x == 0) {
+#pragma unroll
+        for (int w = 0; w < kRedThreads / 32; ++w) {
+            t.loss += sh[w].loss;
+            t.rho += sh[w].rho;
+            t.live += sh[w].live;
+            t.clip += sh[w].clip;
+        }
+    }
+    return t;
 }
 
+// Partial sums of kReduceRowsPerBlock rows per block (2 per thread), so
+// that the dependent fp64 additions per thread stay few and the partial
+// blocks spread over the SMs.
 __global__ void __launch_bounds__(kRedThreads) reduce_partial_kernel(LossWorkspace ws, int64_t N) {
-    __shared__ double shd[kRedThreads];
-    __shared__ long long shl[kRedThreads];
     const int64_t lo = (int64_t)blockIdx.x * kReduceRowsPerBlock;
     const int64_t hi = min(N, lo + kReduceRowsPerBlock);
-    double l = 0.0, rs = 0.0;
-    long long live = 0, clip = 0;
+    LossSums v = {0.0, 0.0, 0, 0};
     for (int64_t i = lo + threadIdx.x; i < hi; i += kRedThreads) {
-        l += ws.contrib[i];
-        rs += (double)ws.rho[i];
+        v.loss += ws.contrib[i];
+        v.rho += (double)ws.rho[i];
         const uint8_t f = ws.flag[i];
-        live += (f & 1u);
-        clip += (f >> 1) & 1u;
+        v.live += (f & 1u);
+        v.clip += (f >> 1) & 1u;
     }
-    l = block_sum_fixed(l, shd);
-    rs = block_sum_fixed(rs, shd);
-    live = block_sum_fixed(live, shl);
-    clip = block_sum_fixed(clip, shl);
+    const LossSums t = block_sums_fixed(v);
     if (threadIdx.x == 0) {
-        ws.part_loss[blockIdx.x] = l;
-        ws.part_rho[blockIdx.x] = rs;
-        ws.part_live[blockIdx.x] = live;
-        ws.part_clip[blockIdx.x] = clip;
+        ws.part_loss[blockIdx.x] = t.loss;
+        ws.part_rho[blockIdx.x] = t.rho;
+        ws.part_live[blockIdx.x] = t.live;
+        ws.part_clip[blockIdx.x] = t.clip;
     }
 }
 
 __global__ void __launch_bounds__(kRedThreads) reduce_final_kernel(LossWorkspace ws, float* loss,
                                                                     leap_loss_stats_t* stats, int accumulate) {
-    __shared__ double shd[kRedThreads];
-    __shared__ long long shl[kRedThreads];
-    double l = 0.0, rs = 0.0;
-    long long live = 0, clip = 0;
+    LossSums v = {0.0, 0.0, 0, 0};
     for (int64_t b = threadIdx.x; b < ws.nblk; b += kRedThreads) {
-        l += ws.part_loss[b];
-        rs += ws.part_rho[b];
-        live += ws.part_live[b];
-        clip += ws.part_clip[b];
+        v.loss += ws.part_loss[b];
+        v.rho += ws.part_rho[b];
+        v.live += ws.part_live[b];
+        v.clip += ws.part_clip[b];
     }
-    l = block_sum_fixed(l, shd);
-    rs = block_sum_fixed(rs, shd);
-    live = block_sum_fixed(live, shl);
-    clip = block_sum_fixed(clip, shl);
+    const LossSums t = block_sums_fixed(v);
     if (threadIdx.x == 0) {
-        loss[0] = accumulate ? loss[0] + (float)l : (float)l;
+        loss[0] = accumulate ? loss[0] + (float)t.loss : (float)t.loss;
         if (stats) {
             if (accumulate) {
-                stats->loss_sum += l;
-                stats->rho_sum += rs;
-                stats->live_tokens += live;
-                stats->clipped_tokens += clip;
+                stats->loss_sum += t.loss;
+                stats->rho_sum += t.rho;
+                stats->live_tokens += t.live;
+                stats->clipped_tokens += t.clip;
             } else {
-                stats->loss_sum = l;
-                stats->rho_sum = rs;
-                stats->live_tokens = live;
-                stats->clipped_tokens = clip;
+                stats->loss_sum = t.loss;
+                stats->rho_sum = t.rho;
+                stats->live_tokens = t.live;
+                stats->clipped_tokens = t.clip;
             }
         }
     }
