@@ -267,7 +267,7 @@ static bool loss_params_ok(const leap_loss_params_t* p) {
     if (!p) return false;
     if (!finite(p->eps_low) || !finite(p->eps_high) || p->eps_low < 0.f || p->eps_high < 0.f) return false;
     if (!finite(p->inv_temp) || !(p->inv_temp > 0.f) || !finite(p->grad_scale)) return false;
-    if (p->flags & ~(LEAP_LOSS_ACCUMULATE | LEAP_LOSS_SINGLE_READ)) return false;
+    if (p->flags & ~(LEAP_LOSS_ACCUMULATE | LEAP_LOSS_SINGLE_READ | LEAP_LOSS_INTERLEAVED_ROWS)) return false;
     return true;
 }
 
@@ -290,8 +290,7 @@ leap_status_t leap_grpo_loss_fwd(const leap_loss_params_t* p, const uint16_t* lo
     if (ws_bytes < loss_workspace_bytes(N)) return LEAP_ERR_INVALID_ARG;
     // Rows of at most kShortRowMaxV columns take the short-row kernel whatever
     // the flag (a group of warps holds each row on chip, read once), where the
-    // persistent two-pass kernel's 1,024-thread CTAs would spend most of a
-    // short row in its block reductions.
+    // pipelined kernel's 16 KB staging chunks would be mostly empty.
     const bool single_read = (p->flags & LEAP_LOSS_SINGLE_READ) != 0 || V <= kShortRowMaxV;
     if (dlogits && single_read && (int64_t)V > fused_max_vocab()) return LEAP_ERR_UNSUPPORTED;
     const LossWorkspace ws = carve_loss_workspace(workspace, N);
@@ -315,6 +314,7 @@ leap_status_t leap_grpo_loss_fwd(const leap_loss_params_t* p, const uint16_t* lo
     a.ws_contrib = ws.contrib;
     a.ws_rho = ws.rho;
     a.ws_flag = ws.flag;
+    a.row_streams = (p->flags & LEAP_LOSS_INTERLEAVED_ROWS) ? 2 : 1;
     a.status = status_ptr();
     if (!a.status) return LEAP_ERR_CUDA;
     cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -68,27 +68,49 @@ struct PipeSmem {
     int abort_flag;
 };
 
+// The order in which every role of a CTA visits its rows c, c + G, ... (c =
+// blockIdx.x, G = gridDim.x, n of them): P interleaved streams, stream p
+// holding the p-th run of ceil(n / P) rows, so that row j of the walk is
+// row ((j mod P) ceil(n / P) + j div P) of the CTA, or none past the end.
+template <int P>
+struct RowSeq {
+    int64_t c, G, n, np;
+    __device__ __forceinline__ explicit RowSeq(int64_t N) : c(blockIdx.x), G(gridDim.x) {
+        n = (N - c + G - 1) / G;
+        np = (n + P - 1) / P;
+    }
+    __device__ __forceinline__ int64_t len() const { return np * P; }
+    __device__ __forceinline__ int64_t row(int64_t j) const {
+        if (j >= np * P) return -1;
+        const int64_t idx = (j % P) * np + j / P;
+        return idx < n ? c + idx * G : -1;
+    }
+};
+
 // One producer: copies every chunk of the CTA's live rows, in order, into a
 // ring of S stages; then waits for whatever of its copies is still in flight.
-template <int S, int CV>
+template <int S, int CV, int P>
 __device__ __forceinline__ void pipe_produce(const RowArgs& a, uint4 (*ring)[CV], uint64_t* full,
                                              uint64_t* empty, uint64_t policy, volatile int* abort_flag) {
     constexpr int64_t kPipeChunk = CV * 16;
-    const int64_t G = gridDim.x;
     const int64_t rowbytes = (int64_t)(a.V & ~7) * 2;
     const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
     uint32_t cnt = 0;
     bool go = true;
-    float w_next = a.w[blockIdx.x];     // the next row's weight and id, a row ahead
-    int id_next = a.ids[blockIdx.x];
-    for (int64_t row = blockIdx.x; go && row < a.N; row += G) {
+    const RowSeq<P> seq(a.N);
+    int64_t rn = seq.row(0);
+    float w_next = a.w[rn];     // the next row's weight and id, a row ahead
+    int id_next = a.ids[rn];
+    for (int64_t j = 0; go && j < seq.len(); ++j) {
+        const int64_t row = rn;
         const float wk = w_next;
         const int id = id_next;
-        if (row + G < a.N) {
-            w_next = a.w[row + G];
-            id_next = a.ids[row + G];
+        rn = seq.row(j + 1);
+        if (rn >= 0) {
+            w_next = a.w[rn];
+            id_next = a.ids[rn];
         }
-        if (!(wk != 0.f && id >= 0 && id < a.V)) continue;
+        if (row < 0 || !(wk != 0.f && id >= 0 && id < a.V)) continue;
         const char* src = reinterpret_cast<const char*>(a.logits + row * a.ld);
         for (int64_t k = 0; k < nch; ++k) {
             const uint32_t s = cnt % S, ph = (cnt / S) & 1u;
@@ -121,7 +143,7 @@ __device__ __forceinline__ void pipe_produce(const RowArgs& a, uint4 (*ring)[CV]
     }
 }
 
-template <int NA, int NB, int SA, int SB, int CVA, int CVB>
+template <int NA, int NB, int SA, int SB, int CVA, int CVB, int P>
 __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(RowArgs a) {
     extern __shared__ __align__(128) unsigned char pipe_smem_raw[];
     PipeSmem<NA, SA, SB, CVA, CVB>& sm = *reinterpret_cast<PipeSmem<NA, SA, SB, CVA, CVB>*>(pipe_smem_raw);
@@ -154,15 +176,14 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
     const int tailn = V & 7;
     const int64_t V8f = (int64_t)(V >> 3);             // whole vectors, all bulk-copied
     const int64_t rowbytes = V8f * 16;
-    const int64_t G = gridDim.x;
     const float c1 = a.inv_temp * kLog2e;
 
     if (warp == 0) {
-        if (lane == 0) pipe_produce<SA, CVA>(a, sm.ringA, sm.fullA, sm.emptyA, l2_policy_evict_last(), abort_flag);
+        if (lane == 0) pipe_produce<SA, CVA, P>(a, sm.ringA, sm.fullA, sm.emptyA, l2_policy_evict_last(), abort_flag);
         return;
     }
     if (warp == 1) {
-        if (lane == 0) pipe_produce<SB, CVB>(a, sm.ringB, sm.fullB, sm.emptyB, l2_policy_evict_first(), abort_flag);
+        if (lane == 0) pipe_produce<SB, CVB, P>(a, sm.ringB, sm.fullB, sm.emptyB, l2_policy_evict_first(), abort_flag);
         return;
     }
 
@@ -172,16 +193,20 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
         // loss and hands (K, coef) to group B, while group A goes on to the
         // next row.
         uint32_t li = 0;
-        float w_next = a.w[blockIdx.x];
-        int id_next = a.ids[blockIdx.x];
-        for (int64_t row = blockIdx.x; row < a.N; row += G) {
+        const RowSeq<P> seq(a.N);
+        int64_t rn = seq.row(0);
+        float w_next = a.w[rn];
+        int id_next = a.ids[rn];
+        for (int64_t j = 0; j < seq.len(); ++j) {
+            const int64_t row = rn;
             const float wk = w_next;
             const int id = id_next;
-            if (row + G < a.N) {
-                w_next = a.w[row + G];
-                id_next = a.ids[row + G];
+            rn = seq.row(j + 1);
+            if (rn >= 0) {
+                w_next = a.w[rn];
+                id_next = a.ids[rn];
             }
-            if (!(wk != 0.f && id >= 0 && id < V)) continue;
+            if (row < 0 || !(wk != 0.f && id >= 0 && id < V)) continue;
             float zy = 0.f, old = 0.f, Adv = 0.f;
             if (lane == 0) {
                 zy = bf16_at(a.logits + row * a.ld + id);
@@ -217,16 +242,20 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
         // The next row's weight and id are loaded a row ahead (every role does;
         // with the finishing warp's early loads of the loss inputs, measured
         // 0.914 -> 0.928 of the copy peak).
-        float w_next = a.w[blockIdx.x];
-        int id_next = a.ids[blockIdx.x];
-        for (int64_t row = blockIdx.x; row < a.N; row += G) {
+        const RowSeq<P> seq(a.N);
+        int64_t rn = seq.row(0);
+        float w_next = a.w[rn];
+        int id_next = a.ids[rn];
+        for (int64_t j = 0; j < seq.len(); ++j) {
+            const int64_t row = rn;
             const float wk = w_next;
             const int id = id_next;
-            if (row + G < a.N) {
-                w_next = a.w[row + G];
-                id_next = a.ids[row + G];
+            rn = seq.row(j + 1);
+            if (rn >= 0) {
+                w_next = a.w[rn];
+                id_next = a.ids[rn];
             }
-            if (!(wk != 0.f && id >= 0 && id < V)) continue;
+            if (row < 0 || !(wk != 0.f && id >= 0 && id < V)) continue;
             const uint16_t* zr = a.logits + row * a.ld;
             // Start live row li once group B has finished row li - 2 (the
             // queue slot's release): pass 1 stays at most about one row
@@ -298,16 +327,21 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
     constexpr int kPipeChunkVec = CVB;
     const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
     uint32_t cnt = 0, li = 0;
-    float w_next = a.w[blockIdx.x];
-    int id_next = a.ids[blockIdx.x];
-    for (int64_t row = blockIdx.x; row < a.N; row += G) {
-        uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
+    const RowSeq<P> seq(a.N);
+    int64_t rn = seq.row(0);
+    float w_next = a.w[rn];
+    int id_next = a.ids[rn];
+    for (int64_t j = 0; j < seq.len(); ++j) {
+        const int64_t row = rn;
         const float wk = w_next;
         const int id = id_next;
-        if (row + G < a.N) {
-            w_next = a.w[row + G];
-            id_next = a.ids[row + G];
+        rn = seq.row(j + 1);
+        if (rn >= 0) {
+            w_next = a.w[rn];
+            id_next = a.ids[rn];
         }
+        if (row < 0) continue;
+        uint4* drow = reinterpret_cast<uint4*>(a.dlogits + row * a.ld);
         if (!(wk != 0.f && id >= 0 && id < V)) {
             for (int64_t vi = tb; vi < V8; vi += TB) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
             if (tb == 0) {
@@ -367,9 +401,9 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
     }
 }
 
-template <int NA, int NB, int SA, int SB, int CVA, int CVB>
+template <int NA, int NB, int SA, int SB, int CVA, int CVB, int P = 1>
 cudaError_t launch_pipe_cfg(const RowArgs& a, cudaStream_t s) {
-    auto kern = fused_loss_pipe_kernel<NA, NB, SA, SB, CVA, CVB>;
+    auto kern = fused_loss_pipe_kernel<NA, NB, SA, SB, CVA, CVB, P>;
     const size_t dyn = sizeof(PipeSmem<NA, SA, SB, CVA, CVB>);
     static std::mutex mu;
     static int done_dev = -1;
@@ -413,6 +447,9 @@ cudaError_t launch_pipe_cfg(const RowArgs& a, cudaStream_t s) {
 // with it 0.840, group A of 8 warps 0.918), but the multi-turn step (long
 // masked runs) 0.904 -> 0.890 as pass 1 ran further ahead of pass 2; with
 // pass 1's lead bounded to two rows of queue: 0.933 and 0.910.
+// Rows visited as P interleaved streams (RowSeq): P = 1 / 2 / 4 single-turn
+// 0.933 / 0.930 / 0.922, multi-turn 0.907 / 0.923 / 0.923; P = 2 is the
+// LEAP_LOSS_INTERLEAVED_ROWS hint, P = 1 the default.
 constexpr int kPipeWarpsA = 4, kPipeWarpsB = 8, kPipeStagesA = 3, kPipeStagesB = 11;
 constexpr int kPipeChunkVectors = 1024;   // 16 KB per staged chunk
 
@@ -420,6 +457,9 @@ constexpr int kPipeChunkVectors = 1024;   // 16 KB per staged chunk
 
 cudaError_t launch_pipe_loss(const RowArgs& a, cudaStream_t s) {
     if (a.N == 0) return cudaSuccess;
+    if (a.row_streams == 2)
+        return launch_pipe_cfg<kPipeWarpsA, kPipeWarpsB, kPipeStagesA, kPipeStagesB, kPipeChunkVectors,
+                               kPipeChunkVectors, 2>(a, s);
     return launch_pipe_cfg<kPipeWarpsA, kPipeWarpsB, kPipeStagesA, kPipeStagesB, kPipeChunkVectors,
                            kPipeChunkVectors>(a, s);
 }

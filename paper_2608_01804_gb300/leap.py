@@ -38,6 +38,7 @@ LEAP_AGG_SEQ_MEAN_TOKEN_MEAN = 0
 LEAP_AGG_TOKEN_MEAN = 1
 LEAP_LOSS_ACCUMULATE = 1
 LEAP_LOSS_SINGLE_READ = 2
+LEAP_LOSS_INTERLEAVED_ROWS = 4
 LEAP_LMHEAD_DHIDDEN = 1
 LEAP_LMHEAD_DW = 2
 LEAP_PASS_BUCKETS = 10
@@ -290,7 +291,7 @@ def loss_workspace(N, V, device):
 def leap_grpo_loss_fwd(logits, ids, old_logp, adv, w, *, V=None, eps_low=0.2, eps_high=0.2, inv_temp=1.0,
                        grad_scale=1.0, accumulate=False, loss=None, logp=None, lse=None, ell=None,
                        dlogits=None, want_dlogits=True, want_outputs=True, workspace=None, stats=None,
-                       single_read=False, stream=None):
+                       single_read=False, interleaved_rows=False, stream=None):
     """Clipped-surrogate loss (and fused dlogits).  Returns a dict of tensors."""
     lp, ld, V = _logits_args(logits, V)
     N = logits.shape[0]
@@ -304,7 +305,8 @@ def leap_grpo_loss_fwd(logits, ids, old_logp, adv, w, *, V=None, eps_low=0.2, ep
         dlogits = torch.empty_like(logits)
     if workspace is None:
         workspace = loss_workspace(N, V, logits.device)
-    flags = (LEAP_LOSS_ACCUMULATE if accumulate else 0) | (LEAP_LOSS_SINGLE_READ if single_read else 0)
+    flags = ((LEAP_LOSS_ACCUMULATE if accumulate else 0) | (LEAP_LOSS_SINGLE_READ if single_read else 0) |
+             (LEAP_LOSS_INTERLEAVED_ROWS if interleaved_rows else 0))
     p = LossParams(eps_low, eps_high, inv_temp, grad_scale, flags)
     st = lib().leap_grpo_loss_fwd(ctypes.byref(p), lp, ld, _ptr(ids), _ptr(old_logp), _ptr(adv), _ptr(w), N, V,
                                   _ptr(loss), _ptr(logp), _ptr(lse), _ptr(ell),

@@ -80,12 +80,14 @@ class GrpoStep:
                                        self.rank_out["turn_adv"], self.rank_out["T_eff"], self.L, self.totals,
                                        M=b.M, agg=self.agg, adv=self.adv, w=self.w)
 
-    def loss_pass(self, logits, ids, old_logp, dlogits, row0=0, accumulate=False, stats=None):
+    def loss_pass(self, logits, ids, old_logp, dlogits, row0=0, accumulate=False, stats=None,
+                  interleaved_rows=False):
         """Step 5 over rows [row0, row0 + logits.shape[0]) of the packed stream."""
         n = logits.shape[0]
         return L.leap_grpo_loss_fwd(logits, ids, old_logp, self.adv[row0:row0 + n], self.w[row0:row0 + n],
                                     V=self.V, loss=self.loss, dlogits=dlogits, want_outputs=False,
-                                    workspace=self.workspace, accumulate=accumulate, stats=stats, **self.loss_kw)
+                                    workspace=self.workspace, accumulate=accumulate, stats=stats,
+                                    interleaved_rows=interleaved_rows, **self.loss_kw)
 
     def run(self, logits, ids, old_logp, dlogits, pg=None):
         """The whole pass for a batch whose logits are all resident."""
@@ -100,12 +102,16 @@ class GrpoStep:
         consecutive row ranges [row0, row0 + logits.shape[0]) that cover the
         stream in order; ids and old_logp are device tensors of all rows.  The
         advantages and weights are computed once for the whole stream, then
-        the fused loss runs chunk by chunk, accumulating the loss."""
+        the fused loss runs chunk by chunk, accumulating the loss.  A packed
+        stream holds long runs of masked rows (prompts, environment feedback),
+        so the loss visits each SM's rows as two interleaved halves
+        (LEAP_LOSS_INTERLEAVED_ROWS)."""
         self.advantages(pg)
         for c, (row0, z, dl) in enumerate(chunks):
             n = z.shape[0]
             self._ensure_workspace(n)
-            self.loss_pass(z, ids[row0:row0 + n], old_logp[row0:row0 + n], dl, row0=row0, accumulate=c > 0)
+            self.loss_pass(z, ids[row0:row0 + n], old_logp[row0:row0 + n], dl, row0=row0, accumulate=c > 0,
+                           interleaved_rows=True)
         return self.loss
 
     def capture(self, logits, ids, old_logp, dlogits, warmup=2):

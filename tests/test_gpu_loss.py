@@ -188,14 +188,38 @@ def test_empty_batch():
     assert loss.item() == 0.0
 
 
+@pytest.mark.parametrize("V", [8193, 8200, 16384, 16392, 24583])
+def test_default_fused_kernel_chunk_boundaries(V):
+    """Vocabularies just past the short-row limit and around the pipelined
+    kernel's 16 KB (8,192-logit) staging chunks: one whole chunk plus a
+    partial vector (8,193), a 16-byte last chunk (8,200), exactly two chunks
+    (16,384), two chunks and one vector (16,392), a ragged third chunk with a
+    partial vector (24,583); every row against the oracle."""
+    L = leap()
+    L.leap_get_device_status()
+    N = 300
+    ld = (V + 7) // 8 * 8
+    z, ids, old, adv, w = _inputs(N, V, seed=V % 61, sigma=3.0, spikes=0.01, ld=ld, old_sigma=0.3)
+    ids[:4] = torch.tensor([0, V - 1, 8191 % V, 8192 % V], dtype=torch.int32, device="cuda")
+    w[:4] = 0.1
+    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V)
+    assert L.leap_get_device_status() == 0
+    rows = list(range(N))
+    orc = _oracle_rows(z, ids, old, adv, w, rows, V)
+    _check_rows(out, orc, rows, V, dl=out["dlogits"])
+    assert abs(out["loss"].item() - orc["loss"]) <= TOL_LOSS_REL * abs(orc["loss"])
+
+
 @pytest.mark.parametrize("N,pattern", [(1, "live"), (151, "random"), (152, "masked"), (153, "runs"),
                                        (1000, "live"), (3001, "runs"), (3001, "random"), (5000, "head")])
-def test_default_fused_kernel_row_partition(N, pattern):
+@pytest.mark.parametrize("interleaved", [False, True])
+def test_default_fused_kernel_row_partition(N, pattern, interleaved):
     """The default fused kernel's persistent CTAs share the rows out among
     themselves and pipeline them (pass 1 of a live row beside pass 2 of the
-    previous one, masked rows in between): every row is written, whatever the
-    pattern of live and masked rows and whether N is below, at or above the
-    CTA count, and the loss equals the oracle's sum over all rows."""
+    previous one, masked rows in between), in order or as two interleaved
+    halves: every row is written, whatever the pattern of live and masked rows
+    and whether N is below, at or above the CTA count, the loss equals the
+    oracle's sum over all rows, and both orders give the same bits."""
     L = leap()
     L.leap_get_device_status()
     V = 9000                                   # above the short-row limit: the pipelined kernel
@@ -205,9 +229,12 @@ def test_default_fused_kernel_row_partition(N, pattern):
             "runs": (r // 97) % 3 != 1, "head": r < N // 7}[pattern]
     w.mul_(torch.as_tensor(keep.astype(np.float32), device="cuda"))
     dl = torch.full_like(z, float("nan"))
-    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, dlogits=dl)
+    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, dlogits=dl, interleaved_rows=interleaved)
     assert L.leap_get_device_status() == 0
     assert not torch.isnan(dl).any()          # every row written
+    if interleaved:                           # the row order changes nothing, bit for bit
+        ref = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V)
+        assert torch.equal(ref["dlogits"], dl) and ref["loss"].item() == out["loss"].item()
     assert torch.all(dl[torch.as_tensor(~keep, device="cuda")] == 0)
     rows = list(range(N))
     orc = _oracle_rows(z, ids, old, adv, w, rows, V)
