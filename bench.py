@@ -990,7 +990,7 @@ def main():
                                                          seg_turn=step.seg_turn).items()}
         dev = dict(logits=logits, ids=ids, old=old, pass_turn=step.pass_turn, num_turns=step.num_turns,
                    seg_offsets=step.seg_offsets, seg_rollout=step.seg_rollout, seg_turn=step.seg_turn)
-        h2d = sum(t.numel() * t.element_size() for t in host.values())
+        small_h2d = sum(t.numel() * t.element_size() for k, t in host.items() if k != "logits")
         loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
         E = max(1, args.e2e_steps)
 
@@ -1015,8 +1015,13 @@ def main():
             t = torch.tensor([e_ms], device=device)
             torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
             e_ms = float(t.item())
+        # run_streamed copies only the logit rows that can carry loss weight (generated turns; the loss
+        # never reads a padding row's logits and writes its dlogits as zeros): the bytes it counted.
+        h2d = small_h2d + step.h2d_logit_bytes
         e2e = {"value": n_valid * world / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": 4, "ms_per_step": e_ms, "steps": E}
+               "d2h_bytes_per_step": 4, "ms_per_step": e_ms, "steps": E,
+               "h2d_logit_rows_per_step": step.h2d_logit_bytes // (logits.shape[1] * logits.element_size()),
+               "note": "logits of rows that cannot carry loss weight (padding) stay on the host"}
         del host
 
     rows = None

@@ -138,7 +138,29 @@ class GrpoStep:
             self.run(logits, ids, old_logp, dlogits)
         return g
 
-    def run_streamed(self, host_logits, ids, old_logp, dlogits, chunk_rows=4096, pg=None):
+    def weighted_row_runs(self):
+        """Row ranges [a, b) of the packed stream that can carry loss weight:
+        the tokens of generated turns (segments with a turn index).  Every
+        other row (prompt, environment feedback, padding) has w = 0, so the
+        loss never reads its logits; a turn pruned by DCP may still be in a
+        range (its rows are read only if weighted, which they are not)."""
+        if getattr(self, "_runs", None) is None:
+            b = self.b
+            runs = []
+            for s in range(len(b.seg_rollout)):
+                if b.seg_turn[s] < 0:
+                    continue
+                lo, hi = int(b.seg_offsets[s]), int(b.seg_offsets[s + 1])
+                if hi <= lo:
+                    continue
+                if runs and runs[-1][1] == lo:
+                    runs[-1][1] = hi
+                else:
+                    runs.append([lo, hi])
+            self._runs = [tuple(r) for r in runs]
+        return self._runs
+
+    def run_streamed(self, host_logits, ids, old_logp, dlogits, chunk_rows=4096, pg=None, weighted_only=True):
         """The whole pass for a batch whose logits are in pinned host memory.
 
         Chunks of `chunk_rows` rows go to two device staging buffers on a copy
@@ -146,10 +168,17 @@ class GrpoStep:
         (the loss accumulates over chunks with LEAP_LOSS_ACCUMULATE; dlogits
         rows are written in place), so the host-to-device copy of the logits
         hides the compute.  ids and old_logp are device tensors of all rows.
+        With weighted_only (the default) only the rows that can carry loss
+        weight (weighted_row_runs) cross the link: the loss never reads the
+        logits of a row of weight 0, and writes its dlogits row as zeros.
+        self.h2d_logit_bytes holds the logit bytes the call copied.
         """
         if not host_logits.is_pinned():
             raise ValueError("host_logits must be in pinned host memory")
         N, ld = host_logits.shape
+        runs = self.weighted_row_runs() if weighted_only else [(0, N)]
+        row_bytes = ld * host_logits.element_size()
+        self.h2d_logit_bytes = 0
         self._ensure_workspace(min(N, chunk_rows))
         comp = torch.cuda.current_stream(self.dev)
         cs = self._copy_stream()
@@ -165,7 +194,11 @@ class GrpoStep:
             if free[c % 2] is not None:
                 cs.wait_event(free[c % 2])          # the loss that read this buffer is done
             with torch.cuda.stream(cs):
-                buf.copy_(host_logits[a:b], non_blocking=True)
+                for lo, hi in runs:
+                    lo, hi = max(lo, a), min(hi, b)
+                    if lo < hi:
+                        buf[lo - a:hi - a].copy_(host_logits[lo:hi], non_blocking=True)
+                        self.h2d_logit_bytes += (hi - lo) * row_bytes
             copied = torch.cuda.Event()
             copied.record(cs)
             comp.wait_event(copied)
@@ -203,7 +236,7 @@ class GrpoStep:
         b = self.b
         single = pg is None or torch.distributed.get_world_size(pg) == 1
         S = len(b.seg_rollout)
-        if single and S <= self.ONE_LAUNCH_TOKEN_SEGMENTS and 4 * b.n + 4 * (S + 1) + 12 * S <= 48 * 1024:
+        if single and S <= self.ONE_LAUNCH_TOKEN_SEGMENTS and 5 * b.n + 4 * (S + 1) + 17 * S + 16 <= 48 * 1024:
             return 1
         return (1 if b.n <= self.ONE_BLOCK_COUNT_ROLLOUTS else 3) + 1
 

@@ -194,6 +194,47 @@ def test_streamed_step_equals_resident_step():
     torch.cuda.synchronize()
     assert loss_small.item() == loss_str.item()
     assert torch.equal(dl_small, dl_res)
+    # Only rows that can carry weight crossed the link (the padding did not).
+    live = sum(hi - lo for lo, hi in step.weighted_row_runs())
+    assert step.h2d_logit_bytes == live * V * 2 < b.N * V * 2
+    assert live == int((step.w != 0).sum().item())
+    # Copying every row gives the same results.
+    dl_all = torch.full_like(z, 7)
+    loss_all = step.run_streamed(host, ids, old, dl_all, chunk_rows=1500, weighted_only=False).clone()
+    torch.cuda.synchronize()
+    assert step.h2d_logit_bytes == b.N * V * 2
+    assert loss_all.item() == loss_str.item() and torch.equal(dl_all, dl_res)
+
+
+def test_streamed_step_packed_multiturn_stream():
+    """The streamed step on a packed multi-turn stream (masked prompts and
+    environment feedback between generated turns, DCP-pruned groups): only
+    the generated turns' rows are copied, and dlogits equal the resident
+    step's bit for bit."""
+    from paper_2608_01804_gb300.step import GrpoStep
+    b = synth.multiturn_dcp_batch(seed=5, num_prompts=4, G=4, M=3, len_lo=64, len_hi=256, prompt_lo=64,
+                                  prompt_hi=256, tau=(1, 3))
+    V = 9000
+    z = synth.logits(b.N, V, 3.0, 220, "cuda", spike_frac=0.01)
+    ids = synth.token_ids(b.N, V, 221, "cuda")
+    old = torch_logp(z, ids, V) + synth.normal(b.N, 0.05, 222, "cuda")
+    step = GrpoStep(b, V, "cuda", gamma=0.9, tau=(1, 3))
+    dl_res = torch.empty_like(z)
+    loss_res = step.run(z, ids, old, dl_res).clone()
+    host = z.cpu().pin_memory()
+    dl_str = torch.full_like(z, 7)
+    step.run_streamed(host, ids, old, dl_str, chunk_rows=700)
+    torch.cuda.synchronize()
+    assert torch.equal(dl_str, dl_res)
+    runs = step.weighted_row_runs()
+    live = sum(hi - lo for lo, hi in runs)
+    assert step.h2d_logit_bytes == live * V * 2 < b.N * V * 2
+    wmask = (step.w != 0).cpu().numpy()
+    inside = np.zeros(b.N, dtype=bool)
+    for lo, hi in runs:
+        inside[lo:hi] = True
+    assert not (wmask & ~inside).any()            # every weighted row was copied
+    assert loss_res.item() != 0.0
 
 
 def test_graph_replay_equals_eager_step():
