@@ -284,6 +284,7 @@ __device__ __forceinline__ void flush_stats(const RankArgs& a, long long (*sst)[
 // for the generic kernel with J <= 2, 6 for the pair kernel).
 constexpr int kRankMinBlocks = 4;
 constexpr int kPairMinBlocks = 6;
+constexpr int kPairLexiMinBlocks = 4;   // the tie-broken comparator: keys and peer loops need registers
 template <int J, bool LEXI>  // rollouts per lane: G <= 32 * J; tie-broken comparator
 __global__ void __launch_bounds__(256, (J <= 2 ? kRankMinBlocks : 1)) rank_adv_kernel(RankArgs a) {
     const int lane = threadIdx.x & 31;
@@ -509,8 +510,8 @@ __global__ void __launch_bounds__(256, (J <= 2 ? kRankMinBlocks : 1)) rank_adv_k
 // it reads both outcomes with one 2-byte load and writes every output of the
 // pair with one vector store (the turn advantages as M float2), and the tier
 // walk and the discount loops unroll.
-template <int MC>
-__global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs a) {
+template <int MC, bool LEXI = false>
+__global__ void __launch_bounds__(256, LEXI ? kPairLexiMinBlocks : kPairMinBlocks) rank_pair_kernel(RankArgs a) {
     constexpr int J = 2, M = MC;
     const int lane = threadIdx.x & 31;
     const int wib = threadIdx.x >> 5;
@@ -526,6 +527,8 @@ __global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs
     for (int64_t group = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib; group < a.num_groups; group += warps) {
         const int64_t i0 = group * G + 2 * lane;
         int pt[J] = {0, 0}, T[J] = {1, 1};
+        float sp[J] = {0.f, 0.f};
+        int tk[J] = {0, 0};
         if (own) {
             const unsigned p2 = *reinterpret_cast<const uint16_t*>(a.pass_turn + i0);
             const unsigned n2 = *reinterpret_cast<const uint16_t*>(a.num_turns + i0);
@@ -533,6 +536,14 @@ __global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs
             pt[1] = (int8_t)(p2 >> 8);
             T[0] = (int8_t)(n2 & 0xffu);
             T[1] = (int8_t)(n2 >> 8);
+            if (LEXI) {
+                const float2 s2 = *reinterpret_cast<const float2*>(a.speedup + i0);
+                const int2 t2 = *reinterpret_cast<const int2*>(a.ntokens + i0);
+                sp[0] = s2.x;
+                sp[1] = s2.y;
+                tk[0] = t2.x;
+                tk[1] = t2.y;
+            }
         }
         bool valid[J] = {own, own}, bad[J];
         int pt0[J], r[J];
@@ -589,6 +600,89 @@ __global__ void __launch_bounds__(256, kPairMinBlocks) rank_pair_kernel(RankArgs
             nw[j] = incl - eq;
             nb[j] = below - incl;
             d[j] = nw[j] - nb[j];
+        }
+        if constexpr (LEXI) {
+            // Tie-broken comparator (r, then speedup higher, then tokens
+            // fewer): the counts above already hold every peer of another
+            // tier; failures tie among themselves; within a passing tier the
+            // keys decide.
+            __shared__ unsigned long long tkeys[8][64];
+            __shared__ int4 lkeys[8][64];
+            bool nan_key = false;
+#pragma unroll
+            for (int j = 0; j < J; ++j) nan_key |= own && r[j] > 0 && isnan(sp[j]);
+            if (!__any_sync(0xffffffffu, nan_key)) {
+                // Without NaN the order within a tier is total: one 64-bit key
+                // (speedup, -tokens) per passing rollout orders exactly as the
+                // tie-breaks (-0 folded into +0); the keys of tier b fill its
+                // slots [lower, lower + size) in the warp's shared memory.
+                unsigned long long key[J];
+#pragma unroll
+                for (int j = 0; j < J; ++j) {
+                    const unsigned b = __float_as_uint(sp[j] + 0.f);
+                    const unsigned o = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+                    key[j] = ((unsigned long long)o << 32) | ~((unsigned)tk[j] ^ 0x80000000u);
+                }
+                const unsigned lt = (1u << lane) - 1u;
+                int lo[J] = {0, 0}, cnt[J] = {0, 0};
+#pragma unroll
+                for (int b = 1; b <= M; ++b) {
+                    const unsigned b0 = __ballot_sync(0xffffffffu, own && r[0] == b);
+                    const unsigned b1 = __ballot_sync(0xffffffffu, own && r[1] == b);
+                    if (own && (r[0] == b || r[1] == b)) {
+                        const int lower = r[0] == b ? nw[0] : nw[1];   // peers in lower tiers
+                        const int size = __popc(b0) + __popc(b1);
+                        if (r[0] == b) {
+                            tkeys[wib][lower + __popc(b0 & lt)] = key[0];
+                            lo[0] = lower;
+                            cnt[0] = size;
+                        }
+                        if (r[1] == b) {
+                            tkeys[wib][lower + __popc(b0) + __popc(b1 & lt)] = key[1];
+                            lo[1] = lower;
+                            cnt[1] = size;
+                        }
+                    }
+                }
+                __syncwarp();
+#pragma unroll
+                for (int j = 0; j < J; ++j) {
+                    int win = 0, loss = 0;
+                    if (own && r[j] > 0) {
+                        for (int p = lo[j]; p < lo[j] + cnt[j]; ++p) {
+                            const unsigned long long kp = tkeys[wib][p];
+                            win += key[j] > kp;
+                            loss += kp > key[j];
+                        }
+                    }
+                    nw[j] += win;
+                    nb[j] += loss;
+                }
+                __syncwarp();
+            } else {
+                // A NaN speedup compares false both ways: the comparator itself,
+                // peer by peer, over the group's (tier, speedup, tokens).
+#pragma unroll
+                for (int j = 0; j < J; ++j) lkeys[wib][2 * lane + j] = make_int4(r[j], __float_as_int(sp[j]), tk[j], 0);
+                __syncwarp();
+#pragma unroll
+                for (int j = 0; j < J; ++j) nw[j] = nb[j] = 0;
+                for (int p = 0; p < G; ++p) {
+                    const int4 kp = lkeys[wib][p];
+                    const int rj = kp.x, tkj = kp.z;
+                    const float spj = __int_as_float(kp.y);
+#pragma unroll
+                    for (int j = 0; j < J; ++j) {
+                        if (!own || 2 * lane + j == p) continue;
+                        const bool tie_r = r[j] == rj && rj > 0;
+                        nw[j] += (r[j] > rj) || (tie_r && (sp[j] > spj || (sp[j] == spj && tk[j] < tkj)));
+                        nb[j] += (rj > r[j]) || (tie_r && (spj > sp[j] || (spj == sp[j] && tkj < tk[j])));
+                    }
+                }
+                __syncwarp();
+            }
+#pragma unroll
+            for (int j = 0; j < J; ++j) d[j] = nw[j] - nb[j];
         }
         const int dd = __reduce_add_sync(0xffffffffu, own ? d[0] * d[0] + d[1] * d[1] : 0);
 
@@ -1173,9 +1267,11 @@ cudaError_t launch_pair(const RankArgs& a, cudaStream_t s) {
     const int warps = 8;
     // A persistent grid (the blocks that fit at once) walks the groups: 10 %
     // faster than one block per 8 groups, and one counter flush per block.
+    const int per_sm = a.cmp == 1 ? kPairLexiMinBlocks : kPairMinBlocks;
     const int64_t blocks = std::min<int64_t>(((int64_t)a.num_groups + warps - 1) / warps,
-                                             (int64_t)device_sm_count() * kPairMinBlocks);
-    rank_pair_kernel<MC><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
+                                             (int64_t)device_sm_count() * per_sm);
+    if (a.cmp == 1) rank_pair_kernel<MC, true><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
+    else rank_pair_kernel<MC, false><<<(unsigned)blocks, warps * 32, 0, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -1204,10 +1300,13 @@ cudaError_t launch_rank_advantages(const RankArgs& a, cudaStream_t s) {
     }
     // The pair kernel's vector accesses need 2-byte aligned byte arrays and
     // 8-byte aligned 4-byte arrays (rollout pairs start at even indices).
-    const bool pair = a.cmp == 0 && a.G % 2 == 0 && a.G <= 64 && aligned_to(a.pass_turn, 2) &&
+    // The tie-broken comparator takes it too, with 8-byte aligned speedups and
+    // token counts.
+    const bool pair = a.G % 2 == 0 && a.G <= 64 && aligned_to(a.pass_turn, 2) &&
                       aligned_to(a.num_turns, 2) && aligned_to(a.T_eff, 2) && aligned_to(a.r_out, 2) &&
                       aligned_to(a.n_worse, 8) && aligned_to(a.n_better, 8) && aligned_to(a.R, 8) &&
-                      aligned_to(a.A, 8) && aligned_to(a.turn_adv, 8);
+                      aligned_to(a.A, 8) && aligned_to(a.turn_adv, 8) &&
+                      (a.cmp == 0 || (aligned_to(a.speedup, 8) && aligned_to(a.ntokens, 8)));
     if (pair) {
         switch (a.M) {
             case 1: return launch_pair<1>(a, s);

@@ -360,3 +360,38 @@ def test_quad_pair_and_generic_counters_and_rewards_at_64(M, reward):
             assert np.max(np.abs(res["A"].cpu().numpy() - orc["A"].reshape(-1))) <= TOL_ADV
             ta = res["turn_adv"].cpu().numpy().reshape(-1, M)
             assert np.max(np.abs(ta - orc["turn_adv"].reshape(-1, M))) <= TOL_ADV
+
+
+@pytest.mark.parametrize("G,M,nan", [(64, 3, False), (16, 2, False), (64, 3, True), (2, 1, False)])
+def test_lexi_pair_and_generic_kernels_agree(G, M, nan):
+    """The tie-broken comparator on the pair layout (even G <= 64, 8-byte
+    aligned speedups and token counts) and on the generic kernel (a 4-byte
+    offset on the outputs) give the same bits and equal the oracle, with
+    exact ties, -0 against +0, and (nan) groups holding a NaN speedup."""
+    rng = np.random.default_rng(17 * G + M + nan)
+    groups = 4096 // G + 3
+    n = groups * G
+    nt = rng.integers(1, M + 1, size=n).astype(np.int8)
+    pt = np.minimum(np.where(rng.random(n) < 0.6, rng.integers(1, M + 1, size=n), 0), nt).astype(np.int8)
+    sp = rng.choice(np.array([0.0, -0.0, 0.5, 1.0, 2.0, np.inf], dtype=np.float32), size=n)
+    tok = rng.choice(np.array([128, 256, 512], dtype=np.int32), size=n)
+    if nan:
+        sp[G * 2 + 1] = np.nan
+        sp[G * 5: G * 5 + G // 2] = np.nan
+    L = leap()
+    dev = torch.device("cuda")
+    args = dict(G=G, M=M, tau_min=0, tau_max=G, gamma=0.8, cmp=L.LEAP_CMP_LEXI, speedup=to_dev(sp, torch.float32),
+                ntokens=to_dev(tok, torch.int32))
+    pt_d, nt_d = to_dev(pt, torch.int8), to_dev(nt, torch.int8)
+    pair = L.leap_group_rank_advantages(pt_d, nt_d, **args)
+    off = lambda k, dt: torch.empty(k + 1, dtype=dt, device=dev)[1:]
+    out = dict(gate=off(groups, torch.uint8), r=off(n, torch.uint8), n_worse=off(n, torch.int32),
+               n_better=off(n, torch.int32), R=off(n, torch.float32), A=off(n, torch.float32),
+               turn_adv=off(n * M, torch.float32), T_eff=off(n, torch.uint8))
+    generic = L.leap_group_rank_advantages(pt_d, nt_d, out=out, **args)
+    torch.cuda.synchronize()
+    for k in pair:
+        assert torch.equal(pair[k], generic[k]), k
+    orc = O.rank_advantages(pt.reshape(-1, G), nt.reshape(-1, G), M, 0, G, 0.8, cmp=O.CMP_LEXI,
+                            speedup=sp.reshape(-1, G), ntokens=tok.reshape(-1, G))
+    _compare(pair, orc, M)
