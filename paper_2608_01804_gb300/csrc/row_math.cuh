@@ -1,7 +1,7 @@
-// Vector helpers of the row kernels (logprob_loss.cu, short_rows.cu): bf16
+// Vector helpers of the row kernels (logprob_loss.cu, loss_pipe.cu, short_rows.cu): bf16
 // vectors of 8 logits as uint4, their masked tail, stores that keep the
 // columns past V, and the per-vector max / exponential-sum / dlogits
-// arithmetic.
+// arithmetic, and the packed fp32x2 instructions (FMA / add / multiply) they use.
 #pragma once
 
 #include "leap_common.cuh"
@@ -39,6 +39,32 @@ __device__ __forceinline__ void store_vec(uint4* drow, int64_t vi, uint4 val, in
     }
 }
 
+// Packed pairs of fp32 (Blackwell's f32x2 FMA / add / multiply: one
+// instruction for two lanes of arithmetic).
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
 __device__ __forceinline__ float bf16_at(const uint16_t* p) {
     return __uint_as_float(((uint32_t)*p) << 16);
 }
@@ -59,33 +85,43 @@ __device__ __forceinline__ float tree_max(const uint4 (&x)[NV]) {
 }
 
 // Sum over NV vectors of 2^(z * c1 - mc), one accumulator per element
-// position (8 independent chains of length NV), then a tree.
+// position (8 independent chains of length NV), then a tree.  Element pairs
+// go through the packed fp32x2 FMA and add (each lane rounds as the scalar
+// instruction would, so the result is the same bits as element by element).
 template <int NV>
 __device__ __forceinline__ float tree_exp_sum(const uint4 (&x)[NV], float c1, float mc) {
-    float acc[8];
+    uint64_t acc[4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) acc[j] = 0.f;
+    for (int q = 0; q < 4; ++q) acc[q] = f2_pack(0.f, 0.f);
+    const uint64_t c12 = f2_pack(c1, c1), nmc2 = f2_pack(-mc, -mc);
 #pragma unroll
     for (int k = 0; k < NV; ++k) {
         const uint32_t w[4] = {x[k].x, x[k].y, x[k].z, x[k].w};
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-            acc[2 * q] += ex2(fmaf(bf16_lo(w[q]), c1, -mc));
-            acc[2 * q + 1] += ex2(fmaf(bf16_hi(w[q]), c1, -mc));
+            float lo, hi;
+            f2_unpack(f2_fma(f2_pack(bf16_lo(w[q]), bf16_hi(w[q])), c12, nmc2), lo, hi);
+            acc[q] = f2_add(acc[q], f2_pack(ex2(lo), ex2(hi)));
         }
     }
-    return ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+    float a[8];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) f2_unpack(acc[q], a[2 * q], a[2 * q + 1]);
+    return ((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]));
 }
 
 // dlogits of one vector: coef * (1[v = y] - 2^(z c1 - K)); `yl` is the target's
-// lane in this vector or -1.
+// lane in this vector or -1.  Element pairs through the packed fp32x2 FMA and
+// multiply (the same bits as element by element).
 __device__ __forceinline__ uint4 dlogit8(const uint4& x, float c1, float K, float coef, int yl) {
     const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+    const uint64_t c12 = f2_pack(c1, c1), nK2 = f2_pack(-K, -K), nc2 = f2_pack(-coef, -coef);
     uint32_t o[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-        float lo = -coef * ex2(fmaf(bf16_lo(w[q]), c1, -K));
-        float hi = -coef * ex2(fmaf(bf16_hi(w[q]), c1, -K));
+        float lo, hi;
+        f2_unpack(f2_fma(f2_pack(bf16_lo(w[q]), bf16_hi(w[q])), c12, nK2), lo, hi);
+        f2_unpack(f2_mul(nc2, f2_pack(ex2(lo), ex2(hi))), lo, hi);
         if (yl == 2 * q) lo += coef;
         if (yl == 2 * q + 1) hi += coef;
         o[q] = pack_bf16x2(lo, hi);
