@@ -1,8 +1,9 @@
 // Fused forward + backward of the clipped surrogate (Eq. 3, KL skipped) with
 // the two passes over a row pipelined across consecutive rows of one SM.
 //
-// One persistent CTA per SM takes rows c, c + G, ... (G = grid size).  Its
-// warps have four roles:
+// One persistent CTA per SM takes its share of the rows: a balanced list
+// (build_row_list: equal live and masked row counts per CTA, in stream order)
+// or rows c, c + G, ... (G = grid size).  Its warps have five roles:
 //   producer A  (one lane)  bulk-copies (TMA, 1-D) each 16 KB chunk of the
 //                           CTA's next live row into ring A (3 stages), an L2
 //                           evict_last policy on the copy so the row stays
@@ -56,6 +57,8 @@ __device__ __forceinline__ void bulk_g2s_hint(void* smem_dst, const void* gsrc, 
         : "memory");
 }
 
+constexpr int kPipeListMax = 576;   // rows per CTA the balanced list holds (fits the shared memory left)
+
 template <int NA, int SA, int SB, int CVA, int CVB>
 struct PipeSmem {
     uint4 ringA[SA][CVA];
@@ -65,39 +68,121 @@ struct PipeSmem {
     float2 kc[2];            // (K = log2 of the row's normaliser in c1 units, coef) per queue slot
     float2 wpart[2][NA];     // per-warp (max, sum) of group A, by row parity
     uint64_t wfull[2], wempty[2];   // group A -> finishing warp, by row parity
+    int32_t list[kPipeListMax];     // this CTA's rows in stream order (balanced assignment)
+    int32_t wcnt[32];               // live rows per warp block while the list is built
+    int32_t nlist;
     int abort_flag;
 };
 
-// The order in which every role of a CTA visits its rows c, c + G, ... (c =
-// blockIdx.x, G = gridDim.x, n of them): P interleaved streams, stream p
-// holding the p-th run of ceil(n / P) rows, so that row j of the walk is
-// row ((j mod P) ceil(n / P) + j div P) of the CTA, or none past the end.
+// The order in which every role of a CTA visits its n rows: the CTA's list
+// (the balanced assignment below) when it has one, else rows c, c + G, ...
+// (c = blockIdx.x, G = gridDim.x); walked as P interleaved streams, stream p
+// holding the p-th run of ceil(n / P) rows, so that row j of the walk is row
+// ((j mod P) ceil(n / P) + j div P) of the CTA, or none past the end.
 template <int P>
 struct RowSeq {
     int64_t c, G, n, np;
-    __device__ __forceinline__ explicit RowSeq(int64_t N) : c(blockIdx.x), G(gridDim.x) {
-        n = (N - c + G - 1) / G;
+    const int32_t* list;
+    __device__ __forceinline__ RowSeq(int64_t N, const int32_t* lst, int32_t nl)
+        : c(blockIdx.x), G(gridDim.x), list(lst) {
+        n = lst ? nl : (N - c + G - 1) / G;
         np = (n + P - 1) / P;
     }
     __device__ __forceinline__ int64_t len() const { return np * P; }
     __device__ __forceinline__ int64_t row(int64_t j) const {
         if (j >= np * P) return -1;
         const int64_t idx = (j % P) * np + j / P;
-        return idx < n ? c + idx * G : -1;
+        if (idx >= n) return -1;
+        return list ? (int64_t)list[idx] : c + idx * G;
     }
 };
 
-// One producer: copies every chunk of the CTA's live rows, in order, into a
-// ring of S stages; then waits for whatever of its copies is still in flight.
+// Balanced assignment of the rows to the G CTAs, built by every CTA from w
+// alone: a live row (w != 0) moves 4V bytes and a masked one 2V, so CTA c
+// takes the live rows of live rank = c (mod G) and the masked rows of masked
+// rank = G - 1 - c (mod G) (the CTAs short of a live row are the ones given an
+// extra masked row), in stream order: every CTA is within one live and one
+// masked row of the average work, where taking rows c, c + G, ... left the
+// busiest CTA 2.5 % above it on the single-turn workload.  Warp k counts the
+// live rows of its block of rows (coalesced loads, ballots), the warps' counts
+// give each block its first live rank, and each warp walks its block again
+// placing this CTA's rows at their index in the list (the number of this
+// CTA's rows of either kind before them).  Needs G >= 32.
+template <int NW>
+__device__ __forceinline__ void build_row_list(const RowArgs& a, int32_t* list, int32_t* wcnt, int32_t* nlist) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t N = a.N;
+    const int G = (int)gridDim.x, c = (int)blockIdx.x;
+    const int64_t per = ((N + NW * 32 - 1) / (NW * 32)) * 32;   // rows per warp block, a multiple of 32
+    const int64_t r0 = (int64_t)warp * per, r1 = r0 + per < N ? r0 + per : N;
+    int cnt = 0;
+    for (int64_t b = r0; b < r1; b += 32 * 8) {
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int64_t r = b + 32 * u + lane;
+            x[u] = r < r1 ? a.w[r] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) cnt += __popc(__ballot_sync(0xffffffffu, x[u] != 0.f));
+    }
+    if (lane == 0) wcnt[warp] = cnt;
+    __syncthreads();
+    int64_t lbefore = 0, ltot = 0;
+    for (int k = 0; k < NW; ++k) {
+        const int v = wcnt[k];
+        ltot += v;
+        if (k < warp) lbefore += v;
+    }
+    // Ranks of the block's first row and their residues mod G, kept up to date
+    // per 32 rows (an increment below 32 <= G needs one conditional subtraction).
+    int64_t lr = lbefore, mr = (r0 < r1 ? r0 : 0) - lbefore;
+    int lrm = (int)(lr % G), mrm = (int)(mr % G);
+    const unsigned lt = (1u << lane) - 1u;
+    for (int64_t b = r0; b < r1; b += 32) {
+        const int64_t r = b + lane;
+        const bool in = r < r1;
+        const bool live = in && a.w[r] != 0.f;
+        const unsigned bal = __ballot_sync(0xffffffffu, live);
+        const int pl = __popc(bal & lt), pm = lane - pl;   // live / masked rows of this chunk before the lane
+        if (in) {
+            int ml = lrm + pl, mm = mrm + pm;
+            if (ml >= G) ml -= G;
+            if (mm >= G) mm -= G;
+            const int64_t my_lr = lr + pl, my_mr = mr + pm;
+            if (live && ml == c)
+                list[(my_lr - c) / G + (my_mr + c) / G] = (int32_t)r;
+            else if (!live && mm == G - 1 - c)
+                list[(my_mr - (G - 1 - c)) / G + (my_lr + G - 1 - c) / G] = (int32_t)r;
+        }
+        const int nin = r1 - b < 32 ? (int)(r1 - b) : 32;
+        const int nl = __popc(bal), nm = nin - nl;
+        lr += nl;
+        mr += nm;
+        lrm += nl;
+        if (lrm >= G) lrm -= G;
+        mrm += nm;
+        if (mrm >= G) mrm -= G;
+    }
+    if (threadIdx.x == 0) {
+        const int64_t mtot = N - ltot;
+        *nlist = (int32_t)((ltot + G - 1 - c) / G + (mtot + c) / G);
+    }
+}
+
+// One producer: copies every chunk of the CTA's live rows, in the CTA's row
+// order, into a ring of S stages; then waits for whatever of its copies is
+// still in flight.
 template <int S, int CV, int P>
 __device__ __forceinline__ void pipe_produce(const RowArgs& a, uint4 (*ring)[CV], uint64_t* full,
-                                             uint64_t* empty, uint64_t policy, volatile int* abort_flag) {
+                                             uint64_t* empty, uint64_t policy, volatile int* abort_flag,
+                                             const int32_t* list, int32_t nlist) {
     constexpr int64_t kPipeChunk = CV * 16;
     const int64_t rowbytes = (int64_t)(a.V & ~7) * 2;
     const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
     uint32_t cnt = 0;
     bool go = true;
-    const RowSeq<P> seq(a.N);
+    const RowSeq<P> seq(a.N, list, nlist);
     int64_t rn = seq.row(0);
     float w_next = a.w[rn];     // the next row's weight and id, a row ahead
     int id_next = a.ids[rn];
@@ -169,7 +254,15 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
         }
         fence_mbar_init();
     }
+    // The balanced row list, for rows visited in order, when the grid is wide
+    // and the list fits (single-turn workload: 0.932 -> 0.936 of the copy
+    // peak; with the interleaved halves of a packed multi-turn stream it
+    // measured 0.933 -> 0.920, so those keep rows c, c + G, ...).
+    const bool listed = P == 1 && gridDim.x >= 32 && (a.N + gridDim.x - 1) / gridDim.x + 2 <= kPipeListMax;
+    if (listed) build_row_list<3 + NA + NB>(a, sm.list, sm.wcnt, &sm.nlist);
     __syncthreads();
+    const int32_t* list = listed ? sm.list : nullptr;
+    const int32_t nlist = listed ? sm.nlist : 0;
 
     const int V = a.V;
     const int64_t V8 = ((int64_t)V + 7) >> 3;
@@ -179,11 +272,13 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
     const float c1 = a.inv_temp * kLog2e;
 
     if (warp == 0) {
-        if (lane == 0) pipe_produce<SA, CVA, P>(a, sm.ringA, sm.fullA, sm.emptyA, l2_policy_evict_last(), abort_flag);
+        if (lane == 0) pipe_produce<SA, CVA, P>(a, sm.ringA, sm.fullA, sm.emptyA, l2_policy_evict_last(), abort_flag, list,
+                                                 nlist);
         return;
     }
     if (warp == 1) {
-        if (lane == 0) pipe_produce<SB, CVB, P>(a, sm.ringB, sm.fullB, sm.emptyB, l2_policy_evict_first(), abort_flag);
+        if (lane == 0) pipe_produce<SB, CVB, P>(a, sm.ringB, sm.fullB, sm.emptyB, l2_policy_evict_first(), abort_flag, list,
+                                                 nlist);
         return;
     }
 
@@ -193,7 +288,7 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
         // loss and hands (K, coef) to group B, while group A goes on to the
         // next row.
         uint32_t li = 0;
-        const RowSeq<P> seq(a.N);
+        const RowSeq<P> seq(a.N, list, nlist);
         int64_t rn = seq.row(0);
         float w_next = a.w[rn];
         int id_next = a.ids[rn];
@@ -242,7 +337,7 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
         // The next row's weight and id are loaded a row ahead (every role does;
         // with the finishing warp's early loads of the loss inputs, measured
         // 0.914 -> 0.928 of the copy peak).
-        const RowSeq<P> seq(a.N);
+        const RowSeq<P> seq(a.N, list, nlist);
         int64_t rn = seq.row(0);
         float w_next = a.w[rn];
         int id_next = a.ids[rn];
@@ -327,7 +422,7 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
     constexpr int kPipeChunkVec = CVB;
     const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
     uint32_t cnt = 0, li = 0;
-    const RowSeq<P> seq(a.N);
+    const RowSeq<P> seq(a.N, list, nlist);
     int64_t rn = seq.row(0);
     float w_next = a.w[rn];
     int id_next = a.ids[rn];
@@ -405,6 +500,7 @@ template <int NA, int NB, int SA, int SB, int CVA, int CVB, int P = 1>
 cudaError_t launch_pipe_cfg(const RowArgs& a, cudaStream_t s) {
     auto kern = fused_loss_pipe_kernel<NA, NB, SA, SB, CVA, CVB, P>;
     const size_t dyn = sizeof(PipeSmem<NA, SA, SB, CVA, CVB>);
+    static_assert(sizeof(PipeSmem<NA, SA, SB, CVA, CVB>) <= 232448, "dynamic shared memory above 227 KB");
     static std::mutex mu;
     static int done_dev = -1;
     int dev = 0;
