@@ -811,7 +811,7 @@ def short_rows(args):
     short vocabularies, through the default entry point and with
     LEAP_LOSS_SINGLE_READ: --warmup untimed calls, then --steps timed ones of
     each, each after an L2 flush; one JSON line per (V, rows).  Rows of
-    V <= 8,192 take the single-read kernel either way."""
+    V <= 32,768 take the short-row kernel either way."""
     from paper_2608_01804_gb300 import build
     build.build()
     from paper_2608_01804_gb300 import leap as L
@@ -820,7 +820,8 @@ def short_rows(args):
     stream = torch.cuda.current_stream()
     flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device=device)
     peak, _ = measured_peaks()
-    cases = [(1024, 16384), (1024, 262144), (4096, 65536), (8192, 32768), (16384, 16384), (32768, 8192)]
+    cases = [(1024, 16384), (1024, 262144), (1000, 262144), (4096, 65536), (8192, 32768), (16384, 16384), (32000, 8192),
+             (32768, 8192), (65536, 4096)]
     if args.short_case:
         cases = [tuple(int(x) for x in args.short_case.split("x"))]
     for Vs, N in cases:

@@ -104,7 +104,7 @@ cudaError_t launch_split_bwd(const RowArgs& a, cudaStream_t s);
 // on each SM through bulk-copy rings (loss_pipe.cu).
 cudaError_t launch_pipe_loss(const RowArgs& a, cudaStream_t s);
 // Fused forward + backward for rows of V <= kShortRowMaxV (short_rows.cu).
-constexpr int32_t kShortRowMaxV = 8192;
+constexpr int32_t kShortRowMaxV = 32768;
 cudaError_t launch_short_row_loss(const RowArgs& a, cudaStream_t s);
 cudaError_t launch_loss_reduce(const LossWorkspace& ws, int64_t N, float* loss, void* stats,
                                bool accumulate, cudaStream_t s);

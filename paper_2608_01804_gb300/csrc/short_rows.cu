@@ -1,6 +1,6 @@
-// Fused forward + backward of the clipped surrogate (Eq. 3) for short rows
-// (V <= 8,192): every leap_grpo_loss_fwd call with dlogits and such a
-// vocabulary lands here (logprob_loss.cu routes it).
+// Fused forward + backward of the clipped surrogate (Eq. 3) for short and
+// mid-size rows (V <= 32,768): every leap_grpo_loss_fwd call with dlogits and
+// such a vocabulary lands here (logprob_loss.cu routes it).
 #include "../../include/leap.h"
 #include "leap_common.cuh"
 #include "leap_internal.h"
@@ -15,47 +15,56 @@ namespace leap {
 namespace {
 
 // ---------------------------------------------------------------------------
-// Fused forward + backward for short rows (V <= 8,192).  A row group of W
-// warps owns one row at a time; warp w of the group owns the contiguous slice
-// of 16-byte vectors [128 w, 128 (w + 1)) of the row (2 KB), lane l vectors
-// 128 w + l + 32 k (k < 4), so the row is read from HBM once.
+// Fused forward + backward for rows of V <= 32,768.  A row group of W warps
+// owns one row at a time; warp w of the group owns the contiguous slice of
+// 16-byte vectors [32 NV w, 32 NV (w + 1)) of the row (512 NV bytes), lane l
+// vectors 32 NV w + l + 32 k (k < NV), so the row is read from HBM once.
+// Shapes (W warps per row, NV vectors per lane, CTA threads, CTAs per SM):
+//   V <= 8,192:   W = 1, 2, 4 or 8, NV = 4, 256 threads, 3 per SM;
+//   V <= 16,384:  W = 8,  NV = 8, 256 threads, 2 per SM;
+//   V <= 32,768:  W = 16, NV = 8, 512 threads, 1 per SM.
 //   * Staging: each warp double-buffers its slice in shared memory.  While it
 //     works on row i, a 1-D bulk copy (TMA) of its slice of row i + 1 is in
 //     flight into the other stage, completing on that stage's mbarrier; every
-//     wait is bounded (LEAP_DEV_TIMEOUT).  Registers hold one row only.
+//     wait is bounded (LEAP_DEV_TIMEOUT).  Registers hold one row only.  The
+//     dlogits slice goes back the same way: the lanes write it to a shared
+//     buffer and one bulk copy stores it (zeros for masked rows come from a
+//     shared zero slice).  Stage entries past a warp's slice hold -inf and the
+//     row's partial last vector is masked in shared memory, so neither the
+//     loads nor the stores carry per-vector bounds checks.
 //   * Arithmetic: the kernel would otherwise be bound by instruction issue,
 //     so the row max is reduced first (packed bf16 maxima, then the warp), the
 //     exponentials 2^((z - m) c1) are taken once and kept in registers
-//     (32 fp32 per lane), element pairs go through packed fp32x2 FMA / add /
+//     (8 NV fp32 per lane), element pairs go through packed fp32x2 FMA / add /
 //     multiply, and dlogits is one multiply per element.
 //   * W > 1: each warp publishes (max, sum) and, if it holds it, the target
 //     logit in shared memory behind one named barrier per live row (two
 //     alternating slots); every warp then merges the W pairs directly.
-//   * FULL (V a multiple of 1,024): every slice is whole, so the per-vector
-//     bounds and tail checks are compiled out.
+//   * FULL (V = 256 NV W): every slice is whole, with no tail.
 // Row groups are persistent and walk rows g, g + stride, ...  Masked rows are
 // not read.
 // ---------------------------------------------------------------------------
-constexpr int kShortThreads = 256;        // 8 warps per CTA
-constexpr int kShortNV = 4;               // 16-byte vectors per lane and row
-constexpr int kShortVPW = 32 * kShortNV;  // vectors per warp slice (2 KB)
-constexpr int kShortMinBlocks = 3;        // register budget: 80 per thread
-
+// Shared memory of a CTA of NW warps (dynamic: 50 KB at NV = 4, 100 KB at
+// NV = 8 with 8 warps, 197 KB with 16).
+template <int NW, int NV>
 struct ShortSmem {
-    uint4 stage[kShortThreads / 32][2][kShortVPW];   // 32 KB: two 2 KB stages per warp
-    uint64_t full[kShortThreads / 32][2];            // one mbarrier per stage
-    float4 part[2][kShortThreads / 32];              // (max, sum, target logit, holds target) per warp
+    uint4 stage[NW][2][32 * NV];   // two stages per warp
+    uint4 out[NW][32 * NV];        // the warp's dlogits slice on its way to HBM
+    uint4 zeros[32 * NV];          // source of the masked rows' slices
+    uint64_t full[NW][2];          // one mbarrier per stage
+    float4 part[2][NW];            // (max, sum, target logit, holds target) per warp
     int abort_flag;
 };
 
-template <int W, bool FULL>
-__global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kernel(RowArgs a) {
-    constexpr int NV = kShortNV, VPW = kShortVPW, TG = 32 * W, GPB = kShortThreads / TG;
-    __shared__ __align__(128) ShortSmem sm;
+template <int W, int NV, int THREADS, int MINB, bool FULL>
+__global__ void __launch_bounds__(THREADS, MINB) short_row_kernel(RowArgs a) {
+    constexpr int NW = THREADS / 32, VPW = 32 * NV, TG = 32 * W, GPB = THREADS / TG;
+    extern __shared__ __align__(128) unsigned char short_smem_raw[];
+    ShortSmem<NW, NV>& sm = *reinterpret_cast<ShortSmem<NW, NV>*>(short_smem_raw);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int gib = warp / W;                  // row group within the block
     const int wig = warp % W;                  // warp within the row group
-    // 32-bit row and vector indices (N < 2^31 is checked on the host; V8 <= 1,024).
+    // 32-bit row and vector indices (N < 2^31 is checked on the host; V8 <= 4,096).
     const int stride = (int)gridDim.x * GPB;
     const int N = (int)a.N;
     const int V = a.V;
@@ -65,6 +74,11 @@ __global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kern
     const int vbase = wig * VPW;                                  // this warp's first vector
     const int nvec = FULL ? VPW : max(0, min(VPW, V8 - vbase));   // vectors in this warp's slice
     const uint32_t slice_bytes = (uint32_t)nvec * 16u;
+    // The row's partial last vector (V not a multiple of 8) is stored element
+    // by element, the whole vectors before it by one bulk copy.
+    const bool owns_tail = !FULL && tailn != 0 && nvec > 0 && vbase + nvec == V8;
+    const uint32_t store_bytes = (uint32_t)(nvec - (owns_tail ? 1 : 0)) * 16u;
+    const uint64_t policy = l2_policy_evict_first();
 
     if (threadIdx.x == 0) sm.abort_flag = 0;
     if (lane == 0) {
@@ -72,6 +86,14 @@ __global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kern
         mbar_init(&sm.full[warp][1], 1);
         fence_mbar_init();
     }
+    if (!FULL) {   // never written by a copy: reads as -inf
+        for (int li = nvec + lane; li < VPW; li += 32) {
+            sm.stage[warp][0][li] = neg_inf4();
+            sm.stage[warp][1][li] = neg_inf4();
+        }
+    }
+    for (int i = threadIdx.x; i < VPW; i += THREADS) sm.zeros[i] = make_uint4(0, 0, 0, 0);
+    fence_proxy_async_smem();   // the zero slice is read by bulk copies
     __syncthreads();
 
     auto is_live = [&](float wr, int idr) { return wr != 0.f && idr >= 0 && idr < V; };
@@ -119,10 +141,12 @@ __global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kern
         const bool bad = (w0 != 0.f) && (id0 < 0 || id0 >= V);
         uint4* drow = reinterpret_cast<uint4*>(a.dlogits + (int64_t)row * a.ld);
         if (w0 == 0.f || bad) {   // masked row: the same branch in every warp of the group
-#pragma unroll
-            for (int k = 0; k < NV; ++k) {
-                const int vi = vbase + lane + 32 * k;
-                if (FULL || vi < V8) store_vec(drow, vi, make_uint4(0, 0, 0, 0), V8, tailn);
+            if (lane == 0) {
+                if (store_bytes) {
+                    bulk_s2g(drow + vbase, &sm.zeros[0], store_bytes, policy);
+                    bulk_commit();
+                }
+                if (owns_tail) store_vec(drow, V8 - 1, make_uint4(0, 0, 0, 0), V8, tailn);
             }
             if (wig == 0 && lane == 0) {
                 write_masked_outputs(a, row);
@@ -138,16 +162,12 @@ __global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kern
                     pending &= ~(1u << st);
                 }   // else: results undefined (LEAP_DEV_TIMEOUT); the copy stays pending
             }
-#pragma unroll
-            for (int k = 0; k < NV; ++k) {
-                const int li = lane + 32 * k;
-                if (FULL) {
-                    x[k] = sm.stage[warp][st][li];
-                } else {
-                    x[k] = (li < nvec) ? sm.stage[warp][st][li] : neg_inf4();
-                    if (tailn && vbase + li == V8 - 1) mask_tail(x[k], tailn);
-                }
+            if (owns_tail) {   // columns >= V of the last vector read as -inf
+                if (lane == 0) mask_tail(sm.stage[warp][st][nvec - 1], tailn);
+                __syncwarp();
             }
+#pragma unroll
+            for (int k = 0; k < NV; ++k) x[k] = sm.stage[warp][st][lane + 32 * k];
             // The target logit, if it lies in this warp's slice.
             const int yl = id0 - vbase * 8;
             const bool own_y = yl >= 0 && yl < nvec * 8;
@@ -195,17 +215,31 @@ __global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kern
             if (W > 1) {
                 if (lane == 0) sm.part[par][warp] = make_float4(m, ssum, zy, own_y ? 1.f : 0.f);
                 named_bar_sync(1 + gib, TG);
-                float4 p[W];
+                const float4* p = &sm.part[par][gib * W];
+                if (W <= 8) {
+                    float4 q[W];
 #pragma unroll
-                for (int v = 0; v < W; ++v) p[v] = sm.part[par][gib * W + v];
-                mrow = p[0].x;
+                    for (int v = 0; v < W; ++v) q[v] = p[v];
+                    mrow = q[0].x;
 #pragma unroll
-                for (int v = 1; v < W; ++v) mrow = fmaxf(mrow, p[v].x);
-                srow = 0.f;
+                    for (int v = 1; v < W; ++v) mrow = fmaxf(mrow, q[v].x);
+                    srow = 0.f;
 #pragma unroll
-                for (int v = 0; v < W; ++v) {
-                    if (p[v].y != 0.f) srow = fmaf(p[v].y, ex2((p[v].x - mrow) * c1), srow);
-                    if (p[v].w != 0.f) zy = p[v].z;
+                    for (int v = 0; v < W; ++v) {
+                        if (q[v].y != 0.f) srow = fmaf(q[v].y, ex2((q[v].x - mrow) * c1), srow);
+                        if (q[v].w != 0.f) zy = q[v].z;
+                    }
+                } else {   // 16 partials: read twice rather than held in registers
+                    mrow = p[0].x;
+#pragma unroll
+                    for (int v = 1; v < W; ++v) mrow = fmaxf(mrow, p[v].x);
+                    srow = 0.f;
+#pragma unroll 4
+                    for (int v = 0; v < W; ++v) {
+                        const float4 q = p[v];
+                        if (q.y != 0.f) srow = fmaf(q.y, ex2((q.x - mrow) * c1), srow);
+                        if (q.w != 0.f) zy = q.z;
+                    }
                 }
                 wscale = (ssum != 0.f) ? ex2((m - mrow) * c1) : 0.f;
                 par ^= 1;   // live rows alternate slots: a slot is rewritten only after the
@@ -220,26 +254,34 @@ __global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kern
             const uint64_t nf2 = f2_pack(nf, nf);
             const int yv = id0 >> 3;
             const int ylane = id0 & 7;
+            if (lane == 0) bulk_wait_read<0>();   // the previous slice has left the buffer
+            __syncwarp();
 #pragma unroll
             for (int k = 0; k < NV; ++k) {
                 const int vi = vbase + lane + 32 * k;
-                if (FULL || vi < V8) {
-                    uint4 d = make_uint4(0, 0, 0, 0);
-                    if (coef != 0.f) {
-                        float o8[8];
+                uint4 d = make_uint4(0, 0, 0, 0);
+                if (coef != 0.f) {
+                    float o8[8];
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) f2_unpack(f2_mul(e2[k][q], nf2), o8[2 * q], o8[2 * q + 1]);
-                        if (vi == yv) {
+                    for (int q = 0; q < 4; ++q) f2_unpack(f2_mul(e2[k][q], nf2), o8[2 * q], o8[2 * q + 1]);
+                    if (vi == yv) {
 #pragma unroll
-                            for (int j = 0; j < 8; ++j)
-                                if (j == ylane) o8[j] += coef;
-                        }
-                        d = make_uint4(pack_bf16x2(o8[0], o8[1]), pack_bf16x2(o8[2], o8[3]),
-                                       pack_bf16x2(o8[4], o8[5]), pack_bf16x2(o8[6], o8[7]));
+                        for (int j = 0; j < 8; ++j)
+                            if (j == ylane) o8[j] += coef;
                     }
-                    if (FULL) st_stream(drow + vi, d);
-                    else store_vec(drow, vi, d, V8, tailn);
+                    d = make_uint4(pack_bf16x2(o8[0], o8[1]), pack_bf16x2(o8[2], o8[3]),
+                                   pack_bf16x2(o8[4], o8[5]), pack_bf16x2(o8[6], o8[7]));
                 }
+                sm.out[warp][lane + 32 * k] = d;
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                if (store_bytes) {
+                    bulk_s2g(drow + vbase, &sm.out[warp][0], store_bytes, policy);
+                    bulk_commit();
+                }
+                if (owns_tail) store_vec(drow, V8 - 1, sm.out[warp][nvec - 1], V8, tailn);
             }
         }
         // Shift the scalar pipeline by one row.
@@ -250,6 +292,7 @@ __global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kern
         w2 = w3;
         id2 = id3;
     }
+    if (lane == 0) bulk_wait_all<0>();   // the dlogits stores have completed
     // Every copy is waited for before its row is used, so one can still be in
     // flight here only after a wait gave up: wait for it (bounded again) so no
     // copy lands in the shared memory of an exited CTA.
@@ -261,9 +304,11 @@ __global__ void __launch_bounds__(kShortThreads, kShortMinBlocks) short_row_kern
 }
 
 // Persistent grid of the short-row kernel: the CTAs that fit at once (cached
-// per device), at most one row group per row.
-template <int W, bool FULL>
+// per device, with the shared-memory opt-in), at most one row group per row.
+template <int W, int NV, int THREADS, int MINB, bool FULL>
 cudaError_t launch_short_rows(const RowArgs& a, cudaStream_t s) {
+    constexpr size_t smem = sizeof(ShortSmem<THREADS / 32, NV>);
+    static_assert(smem <= 232448, "short-row shared memory exceeds the per-CTA limit");
     static std::mutex mu;
     static int cached_dev = -1, cached_resident = 0;
     int dev = 0;
@@ -273,8 +318,12 @@ cudaError_t launch_short_rows(const RowArgs& a, cudaStream_t s) {
     {
         std::lock_guard<std::mutex> lk(mu);
         if (cached_dev != dev) {
+            e = cudaFuncSetAttribute(short_row_kernel<W, NV, THREADS, MINB, FULL>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e != cudaSuccess) return e;
             int per_sm = 0;
-            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, short_row_kernel<W, FULL>, kShortThreads, 0);
+            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, short_row_kernel<W, NV, THREADS, MINB, FULL>,
+                                                              THREADS, smem);
             if (e != cudaSuccess) return e;
             cached_dev = dev;
             cached_resident = per_sm * device_sm_count();
@@ -282,26 +331,30 @@ cudaError_t launch_short_rows(const RowArgs& a, cudaStream_t s) {
         resident = cached_resident;
     }
     if (resident <= 0) return cudaErrorNotSupported;
-    constexpr int GPB = kShortThreads / (32 * W);
+    constexpr int GPB = THREADS / (32 * W);
     const int64_t blocks = std::min<int64_t>((a.N + GPB - 1) / GPB, (int64_t)resident);
-    short_row_kernel<W, FULL><<<(unsigned)blocks, kShortThreads, 0, s>>>(a);
+    short_row_kernel<W, NV, THREADS, MINB, FULL><<<(unsigned)blocks, THREADS, smem, s>>>(a);
     return cudaGetLastError();
+}
+
+template <int W, int NV, int THREADS, int MINB>
+cudaError_t launch_short_shape(const RowArgs& a, cudaStream_t s) {
+    // Whole slices for every warp (V = 256 NV W): no per-vector bounds checks.
+    if (a.V == W * 256 * NV) return launch_short_rows<W, NV, THREADS, MINB, true>(a, s);
+    return launch_short_rows<W, NV, THREADS, MINB, false>(a, s);
 }
 
 }  // namespace
 
 cudaError_t launch_short_row_loss(const RowArgs& a, cudaStream_t s) {
     if (a.N == 0) return cudaSuccess;
-    const int64_t V8s = ((int64_t)a.V + 7) >> 3;
-    const int W = V8s <= kShortVPW ? 1 : V8s <= 2 * kShortVPW ? 2 : V8s <= 4 * kShortVPW ? 4 : 8;
-    // Whole 2 KB slices for every warp (V = 1,024 W): no per-vector bounds checks.
-    const bool full = a.V == W * 8 * kShortVPW;
-    switch (W) {
-        case 1: return full ? launch_short_rows<1, true>(a, s) : launch_short_rows<1, false>(a, s);
-        case 2: return full ? launch_short_rows<2, true>(a, s) : launch_short_rows<2, false>(a, s);
-        case 4: return full ? launch_short_rows<4, true>(a, s) : launch_short_rows<4, false>(a, s);
-        default: return full ? launch_short_rows<8, true>(a, s) : launch_short_rows<8, false>(a, s);
-    }
+    const int64_t V8s = ((int64_t)a.V + 7) >> 3;   // 16-byte vectors per row
+    if (V8s <= 128) return launch_short_shape<1, 4, 256, 3>(a, s);
+    if (V8s <= 256) return launch_short_shape<2, 4, 256, 3>(a, s);
+    if (V8s <= 512) return launch_short_shape<4, 4, 256, 3>(a, s);
+    if (V8s <= 1024) return launch_short_shape<8, 4, 256, 3>(a, s);
+    if (V8s <= 2048) return launch_short_shape<8, 8, 256, 2>(a, s);
+    return launch_short_shape<16, 8, 512, 1>(a, s);
 }
 
 }  // namespace leap

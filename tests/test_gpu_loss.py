@@ -188,20 +188,48 @@ def test_empty_batch():
     assert loss.item() == 0.0
 
 
-@pytest.mark.parametrize("V", [8193, 8200, 16384, 16392, 24583])
+@pytest.mark.parametrize("V,ld,N", [(8193, 8200, 700), (12000, 12000, 333), (16384, 16384, 700),
+                                    (16385, 16392, 400), (24583, 24584, 333), (32000, 32000, 400),
+                                    (32768, 32768, 400)])
+def test_short_row_kernel_mid_vocab(V, ld, N):
+    """The short-row kernel's mid-size shapes: eight warps of 4 KB slices
+    (8,192 < V <= 16,384, two row groups per SM) and sixteen (16,384 < V <=
+    32,768, one per SM).  Whole slices (16,384; 32,768), a single logit past
+    the last whole slice (8,193; 16,385), ragged last vectors, padded ld, more
+    rows than resident row groups, masked rows, and targets on the 2,048-logit
+    slice boundaries; every row against the oracle."""
+    L = leap()
+    L.leap_get_device_status()
+    z, ids, old, adv, w = _inputs(N, V, seed=V % 59 + 3, sigma=3.0, spikes=0.01, ld=ld, old_sigma=0.3)
+    edges = [0, V - 1, 2047, 2048, 4095 % V, 4096 % V, 14335 % V, 14336 % V, 30719 % V, 30720 % V]
+    ids[:len(edges)] = torch.tensor(edges, dtype=torch.int32, device="cuda")
+    w[:len(edges)] = 0.1
+    dl = torch.full_like(z, 3.0)
+    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, dlogits=dl)
+    assert L.leap_get_device_status() == 0
+    if ld > V:
+        assert torch.all(dl[:, V:] == 3.0)        # columns >= V untouched
+    rows = list(range(N))
+    orc = _oracle_rows(z, ids, old, adv, w, rows, V)
+    _check_rows(out, orc, rows, V, dl=dl)
+    assert abs(out["loss"].item() - orc["loss"]) <= TOL_LOSS_REL * abs(orc["loss"])
+    assert (~orc["live"]).any() and (~orc["active"] & orc["live"]).any()
+
+
+@pytest.mark.parametrize("V", [32769, 32776, 40960, 40968, 49159])
 def test_default_fused_kernel_chunk_boundaries(V):
     """Vocabularies just past the short-row limit and around the pipelined
-    kernel's 16 KB (8,192-logit) staging chunks: one whole chunk plus a
-    partial vector (8,193), a 16-byte last chunk (8,200), exactly two chunks
-    (16,384), two chunks and one vector (16,392), a ragged third chunk with a
-    partial vector (24,583); every row against the oracle."""
+    kernel's 16 KB (8,192-logit) staging chunks: four whole chunks plus a
+    partial vector (32,769), a 16-byte last chunk (32,776), exactly five
+    chunks (40,960), five chunks and one vector (40,968), a ragged sixth chunk
+    with a partial vector (49,159); every row against the oracle."""
     L = leap()
     L.leap_get_device_status()
     N = 300
     ld = (V + 7) // 8 * 8
     z, ids, old, adv, w = _inputs(N, V, seed=V % 61, sigma=3.0, spikes=0.01, ld=ld, old_sigma=0.3)
-    ids[:4] = torch.tensor([0, V - 1, 8191 % V, 8192 % V], dtype=torch.int32, device="cuda")
-    w[:4] = 0.1
+    ids[:6] = torch.tensor([0, V - 1, 8191, 8192, 32767, 32768], dtype=torch.int32, device="cuda")
+    w[:6] = 0.1
     out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V)
     assert L.leap_get_device_status() == 0
     rows = list(range(N))
@@ -222,7 +250,7 @@ def test_default_fused_kernel_row_partition(N, pattern, interleaved):
     oracle's sum over all rows, and both orders give the same bits."""
     L = leap()
     L.leap_get_device_status()
-    V = 9000                                   # above the short-row limit: the pipelined kernel
+    V = 33000                                  # above the short-row limit: the pipelined kernel
     z, ids, old, adv, w = _inputs(N, V, seed=N % 53 + 60, sigma=3.0, spikes=0.01, old_sigma=0.3, mask_frac=0.0)
     r = np.arange(N)
     keep = {"live": np.ones(N, bool), "masked": np.zeros(N, bool), "random": np.random.default_rng(N).random(N) < 0.6,

@@ -2,7 +2,8 @@
 sampling temperature (inv_temp = 0.7) and an asymmetric clip range
 (eps_low = 0.2, eps_high = 0.28), on every kernel that evaluates the loss or
 its gradient: the persistent row-pipelined fused kernel with more rows than CTAs,
-the single-read kernel at short and long rows, the forward-only loss with the
+the short-row kernel at mid-size rows, the single-read kernel at short and long
+rows, the forward-only loss with the
 split backward, and the fused lm-head with dhidden and dW.  Old log-probs are
 drawn around the tempered policy's own log-probs with sigma 0.3, and four
 planted tokens sit beyond each edge and between 1.2 and 1.28 (where only the
@@ -95,6 +96,20 @@ def test_single_read_kernel(V, N):
     L.leap_get_device_status()
     z, ids, old, adv, w = _inputs(N, V, seed=V % 89 + 7)
     out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, single_read=True, **PARAMS)
+    assert L.leap_get_device_status() == 0
+    orc = _oracle(z, ids, old, adv, w, V)
+    _both_edges_crossed(orc, adv)
+    _check(out, orc, V, dl=out["dlogits"])
+
+
+@pytest.mark.parametrize("V,N", [(16384, 700), (32000, 400)])
+def test_short_row_kernel_mid_vocab(V, N):
+    """The short-row kernel's eight- and sixteen-warp row groups (4 KB slices)
+    at both clip edges and the tempered softmax."""
+    L = leap()
+    L.leap_get_device_status()
+    z, ids, old, adv, w = _inputs(N, V, seed=V % 83 + 5)
+    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, **PARAMS)
     assert L.leap_get_device_status() == 0
     orc = _oracle(z, ids, old, adv, w, V)
     _both_edges_crossed(orc, adv)
