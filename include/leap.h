@@ -276,11 +276,11 @@ leap_status_t leap_token_logprobs(
  * CTAs that hold it in registers, so it is read from HBM exactly once whatever
  * else is using L2 (supports V <= 262,144).  The default kernel reads a row
  * twice, the second time from L2, which is faster when the loss pass has the
- * GPU's L2 to itself.  Rows of V <= 8,192 take a third kernel with or without
- * the flag: a group of 1-8 warps holds each row in registers (read once) and
- * reduces it with warp shuffles. */
+ * GPU's L2 to itself.  Rows of V <= 32,768 take a third kernel with or
+ * without the flag: a group of 1-16 warps holds each row in registers (read
+ * once) and reduces it with warp shuffles. */
 #define LEAP_LOSS_SINGLE_READ 2u
-/* A scheduling hint for the default fused kernel (rows of V > 8,192 with
+/* A scheduling hint for the default fused kernel (rows of V > 32,768 with
  * dlogits; ignored elsewhere): each persistent CTA visits its rows as two
  * interleaved halves instead of in order, so that long runs of masked rows
  * (prompts and environment feedback in a packed multi-turn stream) and of

@@ -12,7 +12,7 @@
 //                      exchange one (max, sum) pair through distributed
 //                      shared memory: each row is read from HBM exactly once
 //                      whatever else uses L2 (LEAP_LOSS_SINGLE_READ).
-//   (rows of V <= 8,192 take short_row_kernel in short_rows.cu)
+//   (rows of V <= 32,768 take short_row_kernel in short_rows.cu)
 //   split_bwd_kernel   dlogits from a saved lse: 2V read + 2V written.
 //   reduce kernels     fixed-order fp64 sum of the per-row loss terms.
 #include "../../include/leap.h"
@@ -447,9 +447,9 @@ struct FusedCfg {
 // register budget for three CTAs per SM (51 resident clusters).
 constexpr int kBigStages = 1;
 constexpr int kBigMinBlocks = 3;
-// Rows of V <= 8,192 never reach this kernel (they take short_row_kernel).
+// Rows of V <= 32,768 never reach this kernel (they take short_row_kernel).
 constexpr FusedCfg kFused[] = {
-    {2, 256, 8, 2}, {4, 256, 10, 2}, {8, 256, 10, 2}, {8, 256, 16, 2},
+    {4, 256, 10, 2}, {8, 256, 10, 2}, {8, 256, 16, 2},
 };
 
 template <int C, int T, int NV, int STAGES, int MINB = 1>
@@ -573,7 +573,6 @@ cudaError_t launch_fused_loss(const RowArgs& a, bool single_read, cudaStream_t s
     for (const FusedCfg& c : kFused) {
         const int64_t per = (V8 + c.C - 1) / c.C;
         if (per > (int64_t)c.T * c.NV) continue;
-        if (c.C == 2) return launch_fused_cfg<2, 256, 8, 2, 2>(a, s);
         if (c.C == 4) return launch_fused_cfg<4, 256, 10, 2, 2>(a, s);
         if (c.NV == 10) return launch_fused_cfg<8, 256, 10, kBigStages, kBigMinBlocks>(a, s);
         return launch_fused_cfg<8, 256, 16, 2>(a, s);

@@ -48,8 +48,9 @@ def _check_rows(out, orc, rows, V, dl=None):
                                   (30001, 30008), (60000, 60000), (100000, 100000), (151936, 151936), (151936, 152000),
                                   (200000, 200000)])
 def test_fused_loss_all_rows(V, ld, single_read):
-    """Both fused kernels (the row-pipelined one, and with single_read every
-    cluster configuration, sizes 1, 2, 4, 8), ragged V and padded ld."""
+    """Every fused kernel (the short-row kernel up to V = 32,768, the
+    row-pipelined one above it, and with single_read every cluster
+    configuration above it, 4 and 8 CTAs), ragged V and padded ld."""
     L = leap()
     L.leap_get_device_status()
     N = 64 if V > 50000 else 256
