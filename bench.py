@@ -825,7 +825,7 @@ def short_rows(args):
     if args.short_case:
         cases = [tuple(int(x) for x in args.short_case.split("x"))]
     for Vs, N in cases:
-        z = synth.logits(N, Vs, 2.0, 1, device)
+        z = synth.logits(N, Vs, 2.0, 1, device, ld=(Vs + 7) // 8 * 8)
         ids = synth.token_ids(N, Vs, 2, device)
         old = torch.full((N,), -7.0, device=device)
         adv = synth.normal(N, 1.0, 3, device)

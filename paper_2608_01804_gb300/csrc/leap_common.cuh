@@ -225,28 +225,6 @@ __device__ __forceinline__ void bulk_g2s(void* smem_dst, const void* gsrc, uint3
         : "memory");
 }
 
-// 1-D bulk copy own shared memory -> global (bytes and both addresses
-// multiples of 16) in the issuing thread's bulk-async group, with an L2 cache
-// policy; bulk_commit closes the group.
-__device__ __forceinline__ void bulk_s2g(void* gdst, const void* smem_src, uint32_t bytes, uint64_t policy) {
-    asm volatile("cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;" ::"l"(gdst),
-                 "r"(smem_addr(smem_src)), "r"(bytes), "l"(policy)
-                 : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-// Waits until the issuing thread's bulk groups have read their shared-memory
-// sources (all but the newest N groups).
-template <int N>
-__device__ __forceinline__ void bulk_wait_read() {
-    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
-}
-// Waits until the issuing thread's bulk groups have completed (all but the
-// newest N).
-template <int N>
-__device__ __forceinline__ void bulk_wait_all() {
-    asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
-}
-
 // Asynchronous remote store of two floats into the shared memory of a CTA of
 // this cluster; completion is signalled as 8 bytes of tx on that CTA's mbarrier
 // (no fence: the waiter observes the data through the barrier phase).

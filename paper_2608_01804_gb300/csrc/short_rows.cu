@@ -14,6 +14,28 @@
 namespace leap {
 namespace {
 
+// 1-D bulk copy own shared memory -> global (bytes and both addresses
+// multiples of 16) in the issuing thread's bulk-async group, with an L2 cache
+// policy; bulk_commit closes the group.
+__device__ __forceinline__ void bulk_s2g(void* gdst, const void* smem_src, uint32_t bytes, uint64_t policy) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;" ::"l"(gdst),
+                 "r"(smem_addr(smem_src)), "r"(bytes), "l"(policy)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Waits until the issuing thread's bulk groups have read their shared-memory
+// sources (all but the newest N groups).
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// Waits until the issuing thread's bulk groups have completed (all but the
+// newest N).
+template <int N>
+__device__ __forceinline__ void bulk_wait_all() {
+    asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
+}
+
 // ---------------------------------------------------------------------------
 // Fused forward + backward for rows of V <= 32,768.  A row group of W warps
 // owns one row at a time; warp w of the group owns the contiguous slice of
