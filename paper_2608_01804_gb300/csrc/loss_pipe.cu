@@ -352,6 +352,10 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
             }
             if (row < 0 || !(wk != 0.f && id >= 0 && id < V)) continue;
             const uint16_t* zr = a.logits + row * a.ld;
+            // The row's last, partial vector (not bulk-copied) is loaded now,
+            // so its latency hides behind the row's chunks.
+            uint4 tailx = make_uint4(0, 0, 0, 0);
+            if (tailn && ta == 0) tailx = ld_stream(reinterpret_cast<const uint4*>(zr) + V8f);
             // Start live row li once group B has finished row li - 2 (the
             // queue slot's release): pass 1 stays at most about one row
             // ahead of pass 2, so the rows between them still sit in L2 when
@@ -390,8 +394,8 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
                 }
                 ++cnt;
             }
-            if (ok && tailn && ta == 0) {   // the last, partial vector: not bulk-copied
-                uint4 x[1] = {ld_stream(reinterpret_cast<const uint4*>(zr) + V8f)};
+            if (ok && tailn && ta == 0) {   // the last, partial vector
+                uint4 x[1] = {tailx};
                 mask_tail(x[0], tailn);
                 const float bm = tree_max(x);
                 const float mn = fmaxf(m, bm);
@@ -445,6 +449,8 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
             }
             continue;
         }
+        uint4 tailx = make_uint4(0, 0, 0, 0);   // the partial last vector, loaded ahead of its use
+        if (tailn && tb == 0) tailx = ld_stream(reinterpret_cast<const uint4*>(a.logits + row * a.ld) + V8f);
         const uint32_t q = li & 1u;
         if (!mbar_wait(&sm.kcfull[q], (li >> 1) & 1u, a.status, abort_flag)) break;
         const float2 kc = sm.kc[q];
@@ -484,9 +490,8 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
             ++cnt;
         }
         if (ok && tailn && tb == 0) {
-            uint4 x = ld_stream(reinterpret_cast<const uint4*>(a.logits + row * a.ld) + V8f);
             const uint4 d = (coef == 0.f) ? make_uint4(0, 0, 0, 0)
-                                          : dlogit8(x, c1, K, coef, yv == V8f ? ylane : -1);
+                                          : dlogit8(tailx, c1, K, coef, yv == V8f ? ylane : -1);
             store_vec(drow, V8f, d, V8, tailn);
         }
         __syncwarp();
