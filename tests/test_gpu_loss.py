@@ -217,6 +217,27 @@ def test_short_row_kernel_mid_vocab(V, ld, N):
     assert (~orc["live"]).any() and (~orc["active"] & orc["live"]).any()
 
 
+@pytest.mark.parametrize("V", [1000, 16384, 32000])
+@pytest.mark.parametrize("N", [1, 5])
+def test_short_row_kernel_few_rows(V, N):
+    """Fewer rows than row groups: one CTA with a single row group at work
+    (N = 1), and a handful of rows with one masked, for each shape family."""
+    L = leap()
+    L.leap_get_device_status()
+    ld = (V + 7) // 8 * 8
+    z, ids, old, adv, w = _inputs(N, V, seed=N + V % 31, sigma=3.0, spikes=0.01, ld=ld, old_sigma=0.3, mask_frac=0.0)
+    if N > 1:
+        w[N // 2] = 0.0
+    dl = torch.full_like(z, float("nan"))
+    out = L.leap_grpo_loss_fwd(z, ids, old, adv, w, V=V, dlogits=dl)
+    assert L.leap_get_device_status() == 0
+    assert not torch.isnan(dl[:, :V]).any()
+    rows = list(range(N))
+    orc = _oracle_rows(z, ids, old, adv, w, rows, V)
+    _check_rows(out, orc, rows, V, dl=dl)
+    assert abs(out["loss"].item() - orc["loss"]) <= TOL_LOSS_REL * abs(orc["loss"]) + 1e-12
+
+
 @pytest.mark.parametrize("V", [32769, 32776, 40960, 40968, 49159])
 def test_default_fused_kernel_chunk_boundaries(V):
     """Vocabularies just past the short-row limit and around the pipelined
