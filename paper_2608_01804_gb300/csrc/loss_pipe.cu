@@ -70,30 +70,44 @@ struct PipeSmem {
     uint64_t wfull[2], wempty[2];   // group A -> finishing warp, by row parity
     int32_t list[kPipeListMax];     // this CTA's rows in stream order (balanced assignment)
     int32_t wcnt[32];               // live rows per warp block while the list is built
-    int32_t nlist;
+    int32_t nlist, nlive;           // the list's rows, the live ones first
     int abort_flag;
 };
 
-// The order in which every role of a CTA visits its n rows: the CTA's list
-// (the balanced assignment below) when it has one, else rows c, c + G, ...
-// (c = blockIdx.x, G = gridDim.x); walked as P interleaved streams, stream p
-// holding the p-th run of ceil(n / P) rows, so that row j of the walk is row
-// ((j mod P) ceil(n / P) + j div P) of the CTA, or none past the end.
+// The order in which every role of a CTA visits its n rows.  With the CTA's
+// list (the balanced assignment below) and P = 1: the list's order, the
+// stream's.  With the list and P = 2 (the list then holds the CTA's nl live
+// rows, then its masked ones, each in stream order): the live rows spread
+// evenly over the walk, visit j live iff floor((j + 1) nl / n) > floor(j nl /
+// n), so that on every SM masked rows (dlogits zeros, no reads) sit between
+// the live ones instead of the stream's long runs of either (the packed
+// multi-turn workload: 0.934 -> 0.949 of the copy peak; the padded single-turn
+// batch, with short runs, keeps the stream order: 0.951 against 0.945).
+// Without a list: rows c, c + G, ... (c = blockIdx.x, G = gridDim.x), walked
+// as P interleaved streams, stream p holding the p-th run of ceil(n / P)
+// rows, so that row j of the walk is row ((j mod P) ceil(n / P) + j div P) of
+// the CTA, or none past the end.
 template <int P>
 struct RowSeq {
-    int64_t c, G, n, np;
+    int64_t c, G, n, np, nl;
     const int32_t* list;
-    __device__ __forceinline__ RowSeq(int64_t N, const int32_t* lst, int32_t nl)
-        : c(blockIdx.x), G(gridDim.x), list(lst) {
-        n = lst ? nl : (N - c + G - 1) / G;
+    __device__ __forceinline__ RowSeq(int64_t N, const int32_t* lst, int32_t nlst, int32_t nlv)
+        : c(blockIdx.x), G(gridDim.x), nl(nlv), list(lst) {
+        n = lst ? nlst : (N - c + G - 1) / G;
         np = (n + P - 1) / P;
     }
     __device__ __forceinline__ int64_t len() const { return np * P; }
     __device__ __forceinline__ int64_t row(int64_t j) const {
         if (j >= np * P) return -1;
+        if (list) {
+            if (j >= n) return -1;
+            if (P == 1) return (int64_t)list[j];
+            const int64_t lo = j * nl / n, hi = (j + 1) * nl / n;
+            return hi > lo ? (int64_t)list[lo] : (int64_t)list[nl + j - lo];
+        }
         const int64_t idx = (j % P) * np + j / P;
         if (idx >= n) return -1;
-        return list ? (int64_t)list[idx] : c + idx * G;
+        return c + idx * G;
     }
 };
 
@@ -106,10 +120,13 @@ struct RowSeq {
 // busiest CTA 2.5 % above it on the single-turn workload.  Warp k counts the
 // live rows of its block of rows (coalesced loads, ballots), the warps' counts
 // give each block its first live rank, and each warp walks its block again
-// placing this CTA's rows at their index in the list (the number of this
-// CTA's rows of either kind before them).  Needs G >= 32.
-template <int NW>
-__device__ __forceinline__ void build_row_list(const RowArgs& a, int32_t* list, int32_t* wcnt, int32_t* nlist) {
+// placing this CTA's rows at their index in the list: the number of this
+// CTA's rows of either kind before them, or with SPLIT its live rows first
+// (at their index among its live rows) and its masked rows after them (at
+// their index among its masked rows).  Needs G >= 32.
+template <int NW, bool SPLIT>
+__device__ __forceinline__ void build_row_list(const RowArgs& a, int32_t* list, int32_t* wcnt, int32_t* nlist,
+                                               int32_t* nlive) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t N = a.N;
     const int G = (int)gridDim.x, c = (int)blockIdx.x;
@@ -134,6 +151,7 @@ __device__ __forceinline__ void build_row_list(const RowArgs& a, int32_t* list, 
         ltot += v;
         if (k < warp) lbefore += v;
     }
+    const int64_t ncl = (ltot + G - 1 - c) / G;   // this CTA's live rows
     // Ranks of the block's first row and their residues mod G, kept up to date
     // per 32 rows (an increment below 32 <= G needs one conditional subtraction).
     int64_t lr = lbefore, mr = (r0 < r1 ? r0 : 0) - lbefore;
@@ -151,9 +169,10 @@ __device__ __forceinline__ void build_row_list(const RowArgs& a, int32_t* list, 
             if (mm >= G) mm -= G;
             const int64_t my_lr = lr + pl, my_mr = mr + pm;
             if (live && ml == c)
-                list[(my_lr - c) / G + (my_mr + c) / G] = (int32_t)r;
+                list[SPLIT ? (my_lr - c) / G : (my_lr - c) / G + (my_mr + c) / G] = (int32_t)r;
             else if (!live && mm == G - 1 - c)
-                list[(my_mr - (G - 1 - c)) / G + (my_lr + G - 1 - c) / G] = (int32_t)r;
+                list[SPLIT ? ncl + (my_mr - (G - 1 - c)) / G
+                           : (my_mr - (G - 1 - c)) / G + (my_lr + G - 1 - c) / G] = (int32_t)r;
         }
         const int nin = r1 - b < 32 ? (int)(r1 - b) : 32;
         const int nl = __popc(bal), nm = nin - nl;
@@ -166,7 +185,8 @@ __device__ __forceinline__ void build_row_list(const RowArgs& a, int32_t* list, 
     }
     if (threadIdx.x == 0) {
         const int64_t mtot = N - ltot;
-        *nlist = (int32_t)((ltot + G - 1 - c) / G + (mtot + c) / G);
+        *nlist = (int32_t)(ncl + (mtot + c) / G);
+        *nlive = (int32_t)ncl;
     }
 }
 
@@ -176,13 +196,13 @@ __device__ __forceinline__ void build_row_list(const RowArgs& a, int32_t* list, 
 template <int S, int CV, int P>
 __device__ __forceinline__ void pipe_produce(const RowArgs& a, uint4 (*ring)[CV], uint64_t* full,
                                              uint64_t* empty, uint64_t policy, volatile int* abort_flag,
-                                             const int32_t* list, int32_t nlist) {
+                                             const int32_t* list, int32_t nlist, int32_t nlive) {
     constexpr int64_t kPipeChunk = CV * 16;
     const int64_t rowbytes = (int64_t)(a.V & ~7) * 2;
     const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
     uint32_t cnt = 0;
     bool go = true;
-    const RowSeq<P> seq(a.N, list, nlist);
+    const RowSeq<P> seq(a.N, list, nlist, nlive);
     int64_t rn = seq.row(0);
     float w_next = a.w[rn];     // the next row's weight and id, a row ahead
     int id_next = a.ids[rn];
@@ -254,15 +274,15 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
         }
         fence_mbar_init();
     }
-    // The balanced row list, for rows visited in order, when the grid is wide
-    // and the list fits (single-turn workload: 0.932 -> 0.936 of the copy
-    // peak; with the interleaved halves of a packed multi-turn stream it
-    // measured 0.933 -> 0.920, so those keep rows c, c + G, ...).
-    const bool listed = P == 1 && gridDim.x >= 32 && (a.N + gridDim.x - 1) / gridDim.x + 2 <= kPipeListMax;
-    if (listed) build_row_list<3 + NA + NB>(a, sm.list, sm.wcnt, &sm.nlist);
+    // The balanced row list when the grid is wide and the list fits (single-
+    // turn workload, in stream order: 0.932 -> 0.936 of the copy peak against
+    // rows c, c + G, ...; live rows spread evenly, P = 2: above).
+    const bool listed = gridDim.x >= 32 && (a.N + gridDim.x - 1) / gridDim.x + 2 <= kPipeListMax;
+    if (listed) build_row_list<3 + NA + NB, P == 2>(a, sm.list, sm.wcnt, &sm.nlist, &sm.nlive);
     __syncthreads();
     const int32_t* list = listed ? sm.list : nullptr;
     const int32_t nlist = listed ? sm.nlist : 0;
+    const int32_t nlive = listed ? sm.nlive : 0;
 
     const int V = a.V;
     const int64_t V8 = ((int64_t)V + 7) >> 3;
@@ -273,12 +293,12 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
 
     if (warp == 0) {
         if (lane == 0) pipe_produce<SA, CVA, P>(a, sm.ringA, sm.fullA, sm.emptyA, l2_policy_evict_last(), abort_flag, list,
-                                                 nlist);
+                                                 nlist, nlive);
         return;
     }
     if (warp == 1) {
         if (lane == 0) pipe_produce<SB, CVB, P>(a, sm.ringB, sm.fullB, sm.emptyB, l2_policy_evict_first(), abort_flag, list,
-                                                 nlist);
+                                                 nlist, nlive);
         return;
     }
 
@@ -288,7 +308,7 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
         // loss and hands (K, coef) to group B, while group A goes on to the
         // next row.
         uint32_t li = 0;
-        const RowSeq<P> seq(a.N, list, nlist);
+        const RowSeq<P> seq(a.N, list, nlist, nlive);
         int64_t rn = seq.row(0);
         float w_next = a.w[rn];
         int id_next = a.ids[rn];
@@ -337,7 +357,7 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
         // The next row's weight and id are loaded a row ahead (every role does;
         // with the finishing warp's early loads of the loss inputs, measured
         // 0.914 -> 0.928 of the copy peak).
-        const RowSeq<P> seq(a.N, list, nlist);
+        const RowSeq<P> seq(a.N, list, nlist, nlive);
         int64_t rn = seq.row(0);
         float w_next = a.w[rn];
         int id_next = a.ids[rn];
@@ -426,7 +446,7 @@ __global__ void __launch_bounds__(32 * (3 + NA + NB), 1) fused_loss_pipe_kernel(
     constexpr int kPipeChunkVec = CVB;
     const int64_t nch = (rowbytes + kPipeChunk - 1) / kPipeChunk;
     uint32_t cnt = 0, li = 0;
-    const RowSeq<P> seq(a.N, list, nlist);
+    const RowSeq<P> seq(a.N, list, nlist, nlive);
     int64_t rn = seq.row(0);
     float w_next = a.w[rn];
     int id_next = a.ids[rn];
