@@ -281,12 +281,13 @@ leap_status_t leap_token_logprobs(
  * once) and reduces it with warp shuffles. */
 #define LEAP_LOSS_SINGLE_READ 2u
 /* A scheduling hint for the default fused kernel (rows of V > 32,768 with
- * dlogits; ignored elsewhere): each persistent CTA visits its rows as two
- * interleaved halves instead of in order, so that long runs of masked rows
- * (prompts and environment feedback in a packed multi-turn stream) and of
- * live rows overlap on every SM instead of alternating.  Results are the same
- * bit for bit; measured on the packed multi-turn workload 0.907 -> 0.923 of
- * the copy bandwidth, on a padded single-turn batch 0.933 -> 0.930. */
+ * dlogits; ignored elsewhere): each persistent CTA spreads its live rows
+ * evenly among its masked ones instead of visiting them in stream order, so
+ * that long runs of masked rows (prompts and environment feedback in a packed
+ * multi-turn stream) and of live rows overlap on every SM instead of
+ * alternating.  Results are the same bit for bit; measured on the packed
+ * multi-turn workload 0.934 -> 0.950 of the copy bandwidth, on a padded
+ * single-turn batch (short runs) 0.951 -> 0.945. */
 #define LEAP_LOSS_INTERLEAVED_ROWS 4u
 
 typedef struct {

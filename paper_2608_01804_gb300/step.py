@@ -104,7 +104,7 @@ class GrpoStep:
         advantages and weights are computed once for the whole stream, then
         the fused loss runs chunk by chunk, accumulating the loss.  A packed
         stream holds long runs of masked rows (prompts, environment feedback),
-        so the loss visits each SM's rows as two interleaved halves
+        so the loss spreads each SM's live rows evenly among its masked ones
         (LEAP_LOSS_INTERLEAVED_ROWS)."""
         self.advantages(pg)
         for c, (row0, z, dl) in enumerate(chunks):

@@ -266,8 +266,9 @@ def test_default_fused_kernel_chunk_boundaries(V):
 def test_default_fused_kernel_row_partition(N, pattern, interleaved):
     """The default fused kernel's persistent CTAs share the rows out among
     themselves and pipeline them (pass 1 of a live row beside pass 2 of the
-    previous one, masked rows in between), in order or as two interleaved
-    halves: every row is written, whatever the pattern of live and masked rows
+    previous one, masked rows in between), in stream order or with the live
+    rows spread among the masked ones: every row is written, whatever the
+    pattern of live and masked rows
     and whether N is below, at or above the CTA count, the loss equals the
     oracle's sum over all rows, and both orders give the same bits."""
     L = leap()
