@@ -68,7 +68,7 @@ struct RowArgs {
     float* ws_rho;
     uint8_t* ws_flag;
     unsigned int* status;
-    int32_t row_streams;  // pipelined fused kernel: 1 = rows in order, 2 = two interleaved halves
+    int32_t row_streams;  // pipelined fused kernel: 1 = rows in stream order, 2 = live rows spread among masked
 };
 
 // Workspace carve-up of leap_grpo_loss_fwd.

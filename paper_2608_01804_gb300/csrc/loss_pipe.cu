@@ -2,7 +2,7 @@
 // the two passes over a row pipelined across consecutive rows of one SM.
 //
 // One persistent CTA per SM takes its share of the rows: a balanced list
-// (build_row_list: equal live and masked row counts per CTA, in stream order)
+// (build_row_list: equal live and masked row counts per CTA; RowSeq: order)
 // or rows c, c + G, ... (G = grid size).  Its warps have five roles:
 //   producer A  (one lane)  bulk-copies (TMA, 1-D) each 16 KB chunk of the
 //                           CTA's next live row into ring A (3 stages), an L2
@@ -68,7 +68,7 @@ struct PipeSmem {
     float2 kc[2];            // (K = log2 of the row's normaliser in c1 units, coef) per queue slot
     float2 wpart[2][NA];     // per-warp (max, sum) of group A, by row parity
     uint64_t wfull[2], wempty[2];   // group A -> finishing warp, by row parity
-    int32_t list[kPipeListMax];     // this CTA's rows in stream order (balanced assignment)
+    int32_t list[kPipeListMax];     // this CTA's rows (balanced assignment; RowSeq walks it)
     int32_t wcnt[32];               // live rows per warp block while the list is built
     int32_t nlist, nlive;           // the list's rows, the live ones first
     int abort_flag;
