@@ -85,6 +85,10 @@ def parse_args():
                     help="with --lmhead-tokens: a smaller vocabulary, only for small profiling captures")
     ap.add_argument("--prompts", type=int, default=16,
                     help="prompts per rank (16 = the benchmark workload; fewer only for profiling captures)")
+    ap.add_argument("--oracle-configs", action="store_true",
+                    help="host only: time the oracle on the other workloads (tiny, multi-turn, tournament, "
+                         "lm-head), one JSON line each")
+    ap.add_argument("--oracle-config-one", default="", help=argparse.SUPPRESS)
     return ap.parse_args()
 
 
@@ -377,6 +381,117 @@ def workload_config(prompts, rows, valid, world):
             "read and 9.96 GB of dlogits written per step)", "parallelism": "dp%d" % world}
 
 
+def _oracle_one(name, seconds):
+    """The oracle as it stands on one workload, in this process (its BLAS
+    threads as the environment set them); returns the JSON-ready record."""
+    from oracle import leap_oracle as O
+    from paper_2608_01804_gb300 import synth
+    t_begin = time.perf_counter()
+
+    def rank_tokens(batch):
+        G, M = batch.G, batch.M
+        gate = batch.gate_in
+        orc = O.rank_advantages(batch.pass_turn.reshape(-1, G), batch.num_turns.reshape(-1, G), M, 0, G, 0.9,
+                                gate_in=gate)
+        ta, te = orc["turn_adv"].reshape(-1), orc["T_eff"].reshape(-1)
+        Lc, nv, rv = O.rollout_token_counts(batch.seg_offsets, batch.seg_rollout, batch.seg_turn, te)
+        return O.token_advantages(batch.N, batch.seg_offsets, batch.seg_rollout, batch.seg_turn, ta, te, M, 0,
+                                  Lc, nv, rv)
+
+    def loss_rows(z_bits, ids, old, adv, w):
+        live = np.nonzero(w)[0]
+        z = O.bf16_bits_to_f64(z_bits[live])
+        O.grpo_loss_rows(z, ids[live], old[live], adv[live], w[live])
+        return len(live)
+
+    if name == "tiny":          # 16,384 rows at V = 1,024, timed whole
+        batch = synth.tiny_batch()
+        Vt = 1024
+        z = synth.logits(batch.N, Vt, 2.0, 300, "cpu")
+        ids = synth.token_ids(batch.N, Vt, 301, "cpu")
+        old = (torch_logp(z, ids) + synth.normal(batch.N, 0.05, 302, "cpu")).numpy().astype(np.float64)
+        bits = z.view(torch.int16).numpy().view(np.uint16)
+        t0 = time.perf_counter()
+        adv, w = rank_tokens(batch)
+        valid = loss_rows(bits, ids.numpy().astype(np.int64), old, adv, w)
+        dt = time.perf_counter() - t0
+        return {"config": "tiny: 4 prompts x G=8 x 2 turns x 256 = 16,384 rows, V=1024", "value": valid / dt,
+                "unit": "valid tokens/s", "sample": "the whole step (%d valid tokens), %.1f s" % (valid, dt)}
+    if name == "multiturn":     # rank/token steps on the whole stream, the loss on a sample of its live rows
+        batch = synth.multiturn_dcp_batch()
+        src = 256                                   # logits rows drawn once, reused for every row
+        z = synth.logits(src, V, 3.0, 310, "cpu", spike_frac=0.01)
+        ids_src = synth.token_ids(src, V, 311, "cpu")
+        old_src = (torch_logp(z, ids_src) + synth.normal(src, 0.05, 312, "cpu")).numpy().astype(np.float64)
+        bits = z.view(torch.int16).numpy().view(np.uint16)
+        ids_src = ids_src.numpy().astype(np.int64)
+        t0 = time.perf_counter()
+        adv, w = rank_tokens(batch)
+        t_rt = time.perf_counter() - t0
+        live = np.nonzero(w)[0]
+        done, t_loss = 0, 0.0
+        while t_loss < seconds and done < len(live):
+            rows = live[done:done + 32]
+            k = rows % src
+            t1 = time.perf_counter()
+            O.grpo_loss_rows(O.bf16_bits_to_f64(bits[k]), ids_src[k], old_src[k], adv[rows], w[rows])
+            t_loss += time.perf_counter() - t1
+            done += len(rows)
+        est = t_rt + t_loss / done * len(live)
+        return {"config": "multi-turn DCP: 32 prompts x G=16, M=3, %d rows (%d valid), V=151936" % (batch.N, len(live)),
+                "value": len(live) / est, "unit": "valid tokens/s",
+                "sample": "rank/token oracle on the whole stream (%.1f s) + loss fwd and dlogits of the first %d "
+                          "valid rows (%.1f s), scaled to all %d" % (t_rt, done, t_loss, len(live))}
+    if name == "tournament":    # 65,536 groups x 64, M = 3: groups in order until the time is up
+        pt, nt, _, _ = synth.tournament_outcomes()
+        G, M = 64, 3
+        pt, nt = pt.reshape(-1, G), nt.reshape(-1, G)
+        done, dt, step = 0, 0.0, 1024
+        while dt < seconds and done < pt.shape[0]:
+            t1 = time.perf_counter()
+            O.rank_advantages(pt[done:done + step], nt[done:done + step], M, 50, 56, 0.9)
+            dt += time.perf_counter() - t1
+            done += min(step, pt.shape[0] - done)
+        return {"config": "tournament: 65,536 groups x G=64, M=3", "value": done * G / dt, "unit": "rollouts/s",
+                "sample": "%d groups in blocks of %d, %.1f s" % (done, step, dt)}
+    if name == "lmhead":        # 64 tokens of hidden W^T, loss and dhidden, fp64
+        H, T = 5120, 64
+        rng = np.random.default_rng(320)
+        hidden = rng.standard_normal((T, H))
+        Wm = rng.standard_normal((V, H)) * 0.02
+        ids = rng.integers(0, V, T)
+        old = np.full(T, -12.0)
+        adv = rng.standard_normal(T)
+        w = np.full(T, 1.0 / T)
+        t0 = time.perf_counter()
+        O.lmhead_loss_rows(hidden, Wm, ids, old, adv, w, want_dhidden=True)
+        dt = time.perf_counter() - t0
+        return {"config": "fused lm-head: hidden [65,536 x 5120] x W [151,936 x 5120]", "value": T / dt,
+                "unit": "tokens/s (forward + dhidden)",
+                "sample": "%d tokens (logits, loss, dlogits, dhidden in fp64), %.1f s; the whole 65,536 would take "
+                          "%.0f s" % (T, dt, dt * 65536 / T)}
+    raise ValueError(name)
+
+
+def oracle_configs(args):
+    """The oracle, as it stands, on the other workloads: each measurement in a
+    fresh process, with one BLAS thread and (the lm-head's matrix products)
+    with every core; one JSON line per measurement."""
+    cores = os.cpu_count() or 1
+    runs = [("tiny", 1), ("multiturn", 1), ("tournament", 1), ("lmhead", 1), ("lmhead", cores)]
+    for name, threads in runs:
+        env = dict(os.environ)
+        for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+            env[k] = str(threads)
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-config-one", name,
+                            "--cpu-seconds", str(args.cpu_seconds)], env=env, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError("oracle timing %s failed:\n%s" % (name, r.stderr[-2000:]))
+        rec = json.loads(r.stdout.strip().splitlines()[-1])
+        rec.update({"kind": "oracle", "cores": threads, "cpu_model": _cpu_model()})
+        print(json.dumps(rec), flush=True)
+
+
 def reference_arm(args):
     """The oracle (fp64 CPU) as the reference implementation, timed per step on
     a bounded sample of the same workload; rank 0 only."""
@@ -644,7 +759,7 @@ def measure_rows(device, logits, ids, old, step, peak, reps=5):
 
     eager_ms = back_to_back(lambda: st_t.run(zt, it, ot, dl_t))
     graph_ms = back_to_back(graph.replay)
-    nv_t = valid_tokens(tb)
+    nv_t = int((st_t.w != 0).sum().item())   # weighted tokens: DCP-pruned turns in the layout count none
     rows["step_tiny_16384xV1024_eager_vs_graph"] = {
         "eager_ms": eager_ms, "graph_ms": graph_ms, "launches_per_step": st_t.launches_per_run(),
         "eager_valid_tokens_per_s": nv_t / (eager_ms / 1e3), "graph_valid_tokens_per_s": nv_t / (graph_ms / 1e3),
@@ -880,6 +995,12 @@ def logprobs_only(args):
 
 def main():
     args = parse_args()
+    if args.oracle_config_one:
+        print(json.dumps(_oracle_one(args.oracle_config_one, args.cpu_seconds)), flush=True)
+        return
+    if args.oracle_configs:
+        oracle_configs(args)
+        return
     if args.impl == "reference":
         reference_arm(args)
         return
